@@ -1,0 +1,569 @@
+"""Plain, slow CPU oracle: P simulated processes running the paper's Allreduce.
+
+TEST INFRASTRUCTURE, NOT PRODUCT CODE (see ``oracle/__init__.py``).
+
+Source: D. Kolmakov, X. Zhang, "A Generalization of the Allreduce Operation",
+arXiv 2004.09362.  Section and equation labels below are the paper's own.
+
+Model (Sec. "Communication description via permutations")
+----------------------------------------------------------
+* P processes 0..P-1.  Process j owns the vector V_j = (u_{0,j}, ..., u_{P-1,j}) of P
+  blocks (eq. initial_data).  Blocks are unequal when P does not divide n (the paper
+  assumes u = m/P, Sec. "Communication model"); we use the MPI reduce_scatter split:
+  the first n mod P blocks get one extra element (reading C3).
+* T_P is the cyclic group t_k(x) = x + k mod P with generator c = (0 1 ... P-1)
+  (Table 1a); the placement permutation h is the identity (eq. distr_vector_def,
+  reading C4).
+* A distributed vector t_k q has its block i on process t_k(h(i)) = i + k (eq.
+  distr_vector).  Its *content* says where each block's terms come from: the initial
+  vector t_k q_k holds u_{i,i+k} in block i, so a leaf "k" means "block i comes from
+  process i + k".  Combining two same-placement vectors (eq.
+  distr_vectors_combination) makes a node (own, received).
+* A communication operator t_l moves every block from process x to process x + l
+  (eq. comm_op_0).  All processes send and receive at once.
+
+Schedule (Secs. "Bandwidth-optimal algorithm", "Moving towards latency-optimal
+version", "Latency-optimal version")
+----------------------------------------------------------------------
+* N_0 = P, N_{i+1} = ceil(N_i / 2) (eq. bo_starting_set_size); L = ceil(log2 P) steps
+  bring N to 1.
+* Reduction step i: the vectors with index k in [ceil(N_i/2), N_i - 1] (eq.
+  bo_tx_dist) are moved by t^{-floor(N_i/2)} (eq. bo_dir_perms) and each is combined
+  with the vector that now shares its placement (eqs. bo_step_even, bo_step_odd); when
+  N_i is odd the vector with index 0 (q*) sits the step out.
+* To remove r distribution steps, the reduction phase runs K copies of that schedule,
+  copy s shifted by s (vector indices +s, same operators; eq. var_starting_set and the
+  equations after it), so that it ends with q_Sigma at placements 0..K-1.  Vectors of
+  different copies that have the same placement and the same content are the same
+  vector and are sent and combined once.  q* and q' vectors are never merged even at
+  equal placement (Sec. "Latency-optimal version").  The paper says "double the number
+  of resulting vectors" (2^r); the smallest K that lets the remaining distribution
+  steps finish is K = N_{L-r}, which equals 2^r when P is a power of two (reading C7).
+  r = L (K = P) is the latency-optimal version; r = 0 (K = 1) the bandwidth-optimal one.
+* Distribution phase: the reduction steps i = L-r-1, ..., 0 in reverse, with no
+  combination: the vectors at placements [N_i mod 2, ceil(N_i/2) - 1] are copied by
+  t^{+floor(N_i/2)} (end of Sec. "Bandwidth-optimal algorithm").
+* Result: process x's block b is the vector at placement (x - b) mod P.
+
+Precision: f32 runs in float32 (IEEE round-to-nearest-even, as numpy does it); i32 in
+int32 with two's-complement wraparound; bf16 inputs are widened exactly to float32,
+every partial is float32, and each q_Sigma is rounded to bf16 once, at the end of the
+reduction phase (reading C6).  max/min are exact in every type.
+
+Message sizes: a message element counts the size of the type it travels in: a leaf
+(an input block, not yet combined) travels in the input type, a combined partial in the
+accumulation type (float32 for bf16), a distribution-phase block in the output type.
+"""
+
+from __future__ import annotations
+
+import math
+from dataclasses import dataclass, field
+
+import numpy as np
+
+__all__ = [
+    "OPS", "DTYPES", "ceil_log2", "vector_counts", "block_bounds", "schedule_shape",
+    "ExprTable", "Run", "simulate", "allreduce", "round_to_bf16", "is_bf16_exact",
+    "column_reduce_exact", "kahan_sum_f64", "tree_string", "parse_tree",
+    "eval_tree", "cost_model_time", "optimal_steps",
+]
+
+OPS = ("sum", "max", "min")
+DTYPES = ("f32", "bf16", "i32")
+_ITEMSIZE = {"f32": 4, "bf16": 2, "i32": 4}
+_ACC_ITEMSIZE = {"f32": 4, "bf16": 4, "i32": 4}
+
+
+# ---------------------------------------------------------------------------
+# Schedule arithmetic
+# ---------------------------------------------------------------------------
+
+def ceil_log2(P: int) -> int:
+    """L = ceil(log2 P): the number of reduction steps (Sec. "Bandwidth-optimal
+    algorithm": the reduction phase takes ceil(log P) steps)."""
+    if P < 1:
+        raise ValueError("P must be >= 1")
+    L = 0
+    while (1 << L) < P:
+        L += 1
+    return L
+
+
+def vector_counts(P: int) -> list[int]:
+    """[N_0, ..., N_L] with N_0 = P and N_{i+1} = ceil(N_i / 2) (eq.
+    bo_starting_set_size)."""
+    Ns = [P]
+    while Ns[-1] > 1:
+        Ns.append((Ns[-1] + 1) // 2)
+    return Ns
+
+
+def block_bounds(n: int, P: int) -> list[tuple[int, int]]:
+    """Block i of every vector (eq. initial_data).  The paper assumes equal blocks
+    u = m/P (Sec. "Communication model"); for P not dividing n the first n mod P blocks
+    get one extra element (reading C3)."""
+    q, rem = divmod(n, P)
+    out, start = [], 0
+    for i in range(P):
+        size = q + (1 if i < rem else 0)
+        out.append((start, start + size))
+        start += size
+    assert start == n
+    return out
+
+
+def schedule_shape(P: int, steps: int) -> dict:
+    """Step count S in [L, 2L] (abstract; Sec. "Moving towards latency-optimal
+    version": S = 2 ceil(log P) - r, 0 <= r <= ceil(log P)).  Returns L, S, r and the
+    number K of q_Sigma copies the reduction phase must end with (reading C7:
+    K = N_{L-r})."""
+    L = ceil_log2(P)
+    if not (L <= steps <= 2 * L):
+        raise ValueError(f"steps={steps} outside [{L}, {2 * L}] for P={P}")
+    r = 2 * L - steps
+    K = vector_counts(P)[L - r]
+    return {"P": P, "L": L, "S": steps, "r": r, "K": K}
+
+
+# ---------------------------------------------------------------------------
+# Contents of distributed vectors (symbolic)
+# ---------------------------------------------------------------------------
+
+class ExprTable:
+    """Interned contents.  A leaf k is the initial vector t_k q_k (block i from process
+    i + k, eq. initial_distr_vector); a pair (a, b) is the combination "own (+)
+    received" of two same-placement vectors (eq. distr_vectors_combination)."""
+
+    def __init__(self):
+        self.nodes: list = []          # id -> ("leaf", k) | ("pair", a, b)
+        self._leaf: dict[int, int] = {}
+        self._pair: dict[tuple[int, int], int] = {}
+
+    def leaf(self, k: int) -> int:
+        if k not in self._leaf:
+            self._leaf[k] = len(self.nodes)
+            self.nodes.append(("leaf", k))
+        return self._leaf[k]
+
+    def pair(self, a: int, b: int) -> int:
+        key = (a, b)
+        if key not in self._pair:
+            self._pair[key] = len(self.nodes)
+            self.nodes.append(("pair", a, b))
+        return self._pair[key]
+
+    def is_leaf(self, e: int) -> bool:
+        return self.nodes[e][0] == "leaf"
+
+    def tree(self, e: int):
+        """Nested tuples of leaf offsets."""
+        node = self.nodes[e]
+        if node[0] == "leaf":
+            return node[1]
+        return (self.tree(node[1]), self.tree(node[2]))
+
+    def leaves(self, e: int) -> list[int]:
+        out, stack = [], [e]
+        while stack:
+            node = self.nodes[stack.pop()]
+            if node[0] == "leaf":
+                out.append(node[1])
+            else:
+                stack.append(node[2])
+                stack.append(node[1])
+        return out
+
+
+def tree_string(t) -> str:
+    """'(a+b)' notation for a nested-tuple tree; leaves are integers."""
+    if isinstance(t, int):
+        return str(t)
+    return "(" + tree_string(t[0]) + "+" + tree_string(t[1]) + ")"
+
+
+def parse_tree(s: str):
+    """Inverse of tree_string (used for the hand-derived fixtures in tests/golden)."""
+    s = s.replace(" ", "")
+    pos = 0
+
+    def node():
+        nonlocal pos
+        if s[pos] == "(":
+            pos += 1
+            a = node()
+            assert s[pos] == "+", s
+            pos += 1
+            b = node()
+            assert s[pos] == ")", s
+            pos += 1
+            return (a, b)
+        start = pos
+        while pos < len(s) and s[pos].isdigit():
+            pos += 1
+        return int(s[start:pos])
+
+    t = node()
+    assert pos == len(s), s
+    return t
+
+
+def eval_tree(t, leaf_value, op: str):
+    """Evaluate a nested-tuple tree with leaf_value(k) at the leaves, combining with op
+    in whatever numpy type the leaves carry."""
+    if isinstance(t, int):
+        return leaf_value(t)
+    return _combine(op, eval_tree(t[0], leaf_value, op), eval_tree(t[1], leaf_value, op))
+
+
+def _reduce_partner(x: int, d: int, P: int) -> int:
+    """Where process x sends during a reduction step: the operator t^{-d} moves every
+    block from x to x - d (eqs. comm_op_0, bo_dir_perms)."""
+    return (x - d) % P
+
+
+def _distribute_partner(x: int, d: int, P: int) -> int:
+    """Where process x sends during a distribution step: the reversed operator t^{+d}
+    (end of Sec. "Bandwidth-optimal algorithm")."""
+    return (x + d) % P
+
+
+def _combine(op: str, a, b):
+    """The reduction operator (+) of the Allreduce (Sec. "Combination of distributed
+    data vectors"); elementwise, in the operands' own numpy type."""
+    if op == "sum":
+        return a + b
+    if op == "max":
+        return np.maximum(a, b)
+    if op == "min":
+        return np.minimum(a, b)
+    raise ValueError(op)
+
+
+# ---------------------------------------------------------------------------
+# bf16 rounding (reading C6), written from the format's definition
+# ---------------------------------------------------------------------------
+
+def round_to_bf16(x: np.ndarray) -> np.ndarray:
+    """Round float32 values to the nearest bfloat16 (ties to even), returned as float32.
+    bfloat16 keeps the top 16 bits of the float32 encoding (sign, 8 exponent bits,
+    7 fraction bits); rounding looks at the 16 discarded bits.  Finite inputs only."""
+    x = np.ascontiguousarray(x, dtype=np.float32)
+    bits = x.view(np.uint32).astype(np.uint64)
+    upper = bits >> np.uint64(16)
+    lower = bits & np.uint64(0xFFFF)
+    half = np.uint64(0x8000)
+    round_up = (lower > half) | ((lower == half) & ((upper & np.uint64(1)) == np.uint64(1)))
+    upper = upper + round_up.astype(np.uint64)
+    out = (upper << np.uint64(16)).astype(np.uint32)
+    return out.view(np.float32)
+
+
+def is_bf16_exact(x: np.ndarray) -> bool:
+    x = np.ascontiguousarray(x, dtype=np.float32)
+    return bool(np.all((x.view(np.uint32) & np.uint32(0xFFFF)) == 0))
+
+
+# ---------------------------------------------------------------------------
+# The simulation
+# ---------------------------------------------------------------------------
+
+@dataclass
+class Run:
+    """Everything one simulated Allreduce produced."""
+    P: int
+    n: int
+    steps: int
+    L: int
+    r: int
+    K: int
+    op: str
+    dtype: str
+    exprs: ExprTable
+    outputs: list | None                 # per rank: array over the selected elements
+    out_key: list = field(default_factory=list)   # out_key[x][b] = (placement, expr)
+    log: list = field(default_factory=list)       # one dict per communication step
+    after_reduction: list = field(default_factory=list)  # per shift s: key at placement s
+    states: list = field(default_factory=list)    # per reduction step: per shift: keys
+    combines: list = field(default_factory=list)  # per reduction step: distinct combines
+
+    def output_tree(self, x: int, b: int):
+        return self.exprs.tree(self.out_key[x][b][1])
+
+    def message_elems_per_rank(self, x: int) -> int:
+        """Elements rank x sends over the whole Allreduce."""
+        tot = 0
+        for st in self.log:
+            for (src, _dst, items) in st["messages"]:
+                if src == x:
+                    tot += sum(cnt for (_k, cnt, _sz) in items)
+        return tot
+
+    def message_blocks_per_rank(self, x: int) -> int:
+        tot = 0
+        for st in self.log:
+            for (src, _dst, items) in st["messages"]:
+                if src == x:
+                    tot += len(items)
+        return tot
+
+    def step_bytes(self) -> list[int]:
+        """Bytes sent per communication step, summed over all processes."""
+        return [sum(cnt * sz for (_s, _d, items) in st["messages"] for (_k, cnt, sz) in items)
+                for st in self.log]
+
+
+def simulate(P: int, n: int, steps: int, inputs=None, op: str = "sum",
+             dtype: str = "f32", elements=None) -> Run:
+    """Run the Allreduce schedule with P explicit process stores and explicit
+    per-step message lists.
+
+    inputs: None for a symbolic run (contents and messages only), else a sequence of P
+      1-D numpy arrays of length n (float32 for f32/bf16 -- bf16 values must be exactly
+      representable -- or int32 for i32).
+    elements: optional sorted array of global element indices; the run then carries
+      only those elements (every operation is elementwise, so they come out exactly as
+      in a full run).  Message sizes are always those of the full vectors.
+    """
+    if op not in OPS:
+        raise ValueError(op)
+    if dtype not in DTYPES:
+        raise ValueError(dtype)
+    shape = schedule_shape(P, steps)
+    L, r, K = shape["L"], shape["r"], shape["K"]
+    Ns = vector_counts(P)
+    bounds = block_bounds(n, P)
+    block_len = [hi - lo for (lo, hi) in bounds]
+    ex = ExprTable()
+    itemsize = _ITEMSIZE[dtype]
+    acc_itemsize = _ACC_ITEMSIZE[dtype]
+
+    # Per-block element selection (global indices inside the block).
+    if elements is None:
+        sel = [np.arange(lo, hi, dtype=np.int64) for (lo, hi) in bounds]
+    else:
+        elements = np.asarray(elements, dtype=np.int64)
+        sel = [elements[(elements >= lo) & (elements < hi)] for (lo, hi) in bounds]
+
+    have_values = inputs is not None
+    if have_values:
+        if len(inputs) != P:
+            raise ValueError("need one input vector per process")
+        want = np.int32 if dtype == "i32" else np.float32
+        inputs = [np.asarray(v) for v in inputs]
+        for v in inputs:
+            if v.shape != (n,) or v.dtype != want:
+                raise ValueError(f"input must be shape ({n},) {want}")
+            if dtype == "bf16" and not is_bf16_exact(v):
+                raise ValueError("bf16 inputs must be exactly representable in bf16")
+
+    # --- initial data: Q_initial = t_0 q_0 : t_1 q_1 : ... : t_{P-1} q_{P-1}
+    # (eq. distr_vector_set).  Process x holds block (x - k) mod P of t_k q_k, which is
+    # its own block u_{x-k, x}.
+    store = [dict() for _ in range(P)]
+    for x in range(P):
+        for k in range(P):
+            key = (k, ex.leaf(k))
+            b = (x - k) % P
+            store[x][key] = inputs[x][sel[b]].copy() if have_values else None
+
+    # Each shifted copy s of the schedule starts from the same initial set, its index k
+    # naming the vector at placement s + k (eq. var_starting_set).
+    sched = [[((s + k) % P, ex.leaf((s + k) % P)) for k in range(P)] for s in range(K)]
+    run = Run(P=P, n=n, steps=steps, L=L, r=r, K=K, op=op, dtype=dtype, exprs=ex,
+              outputs=None)
+
+    # --- reduction phase: L steps
+    for i in range(L):
+        N = Ns[i]
+        d = N // 2            # operator t^{-floor(N_i/2)} (eq. bo_dir_perms)
+        c = N - d             # ceil(N_i/2)
+        # Q_TX,i of every shifted copy (eq. bo_tx_dist and its shifted form), each
+        # distinct (placement, content) vector once.
+        tx = []
+        seen = set()
+        for s in range(K):
+            for k in range(c, N):
+                key = sched[s][k]
+                if key not in seen:
+                    seen.add(key)
+                    tx.append(key)
+        # Communication: process x sends its blocks of the TX vectors to x - d.
+        messages = []
+        inbox = [dict() for _ in range(P)]
+        for x in range(P):
+            dst = _reduce_partner(x, d, P)
+            items = []
+            for key in tx:
+                b = (x - key[0]) % P
+                sz = itemsize if ex.is_leaf(key[1]) else acc_itemsize
+                items.append((key, block_len[b], sz))
+                # the block keeps its index; its placement moves by -d
+                moved = ((key[0] - d) % P, key[1])
+                inbox[dst][moved] = store[x][key]
+            messages.append((x, dst, items))
+        run.log.append({"phase": "reduce", "i": i, "N": N, "d": d,
+                        "tx": list(tx), "messages": messages})
+        # Combination (eqs. bo_step_even / bo_step_odd and their shifted forms).
+        new_store = [dict() for _ in range(P)]
+        new_sched = []
+        step_combines = []
+        combined = set()
+        for s in range(K):
+            q = sched[s]
+            nq = []
+            for k in range(c):
+                if k == 0 and N % 2 == 1:
+                    key = q[0]                 # q*: sits this step out
+                    for x in range(P):
+                        new_store[x][key] = store[x][key]
+                else:
+                    own = q[k]
+                    moved = ((q[k + d][0] - d) % P, q[k + d][1])
+                    assert moved[0] == own[0]
+                    key = (own[0], ex.pair(own[1], moved[1]))
+                    if key not in combined:
+                        combined.add(key)
+                        step_combines.append(key)
+                        for x in range(P):
+                            if have_values:
+                                new_store[x][key] = _combine(op, store[x][own], inbox[x][moved])
+                            else:
+                                new_store[x][key] = None
+                nq.append(key)
+            new_sched.append(nq)
+        sched = new_sched
+        store = new_store
+        run.states.append([list(q) for q in sched])
+        run.combines.append(step_combines)
+
+    # --- end of the reduction phase: shift s holds q_Sigma at placement s
+    for s in range(K):
+        assert len(sched[s]) == 1 and sched[s][0][0] == s
+    run.after_reduction = [sched[s][0] for s in range(K)]
+    at_place = {s: sched[s][0] for s in range(K)}
+    if have_values and dtype == "bf16":
+        # one rounding of each result to bf16 (reading C6)
+        for x in range(P):
+            for s in range(K):
+                key = at_place[s]
+                store[x][key] = round_to_bf16(store[x][key])
+
+    # --- distribution phase: reduction steps L-r-1 .. 0 reversed, no combination
+    for i in range(L - r - 1, -1, -1):
+        N = Ns[i]
+        d = N // 2
+        c = N - d
+        senders = list(range(N % 2, c))
+        messages = []
+        inbox = [dict() for _ in range(P)]
+        for x in range(P):
+            dst = _distribute_partner(x, d, P)
+            items = []
+            for p in senders:
+                key = at_place[p]
+                b = (x - p) % P
+                items.append((key, block_len[b], itemsize))
+                inbox[dst][((p + d) % P, key[1])] = store[x][key]
+            messages.append((x, dst, items))
+        run.log.append({"phase": "distribute", "i": i, "N": N, "d": d,
+                        "tx": [at_place[p] for p in senders], "messages": messages})
+        for p in senders:
+            newkey = ((p + d) % P, at_place[p][1])
+            assert (p + d) % P not in at_place
+            at_place[(p + d) % P] = newkey
+            for x in range(P):
+                store[x][newkey] = inbox[x][newkey]
+
+    assert sorted(at_place) == list(range(P))
+
+    # --- result: process x's block b sits at placement (x - b) mod P
+    run.out_key = [[at_place[(x - b) % P] for b in range(P)] for x in range(P)]
+    if have_values:
+        outs = []
+        for x in range(P):
+            parts = [store[x][run.out_key[x][b]] for b in range(P)]
+            outs.append(np.concatenate(parts) if parts else np.zeros(0, inputs[x].dtype))
+        run.outputs = outs
+    return run
+
+
+def allreduce(inputs, steps: int, op: str = "sum", dtype: str = "f32", elements=None):
+    """MPI_Allreduce semantics (Sec. "Introduction"): every process ends with the
+    op-reduction of all P input vectors.  Returns the list of P output arrays (over the
+    selected elements when ``elements`` is given)."""
+    P = len(inputs)
+    n = len(inputs[0]) if P else 0
+    return simulate(P, n, steps, inputs=inputs, op=op, dtype=dtype,
+                    elements=elements).outputs
+
+
+# ---------------------------------------------------------------------------
+# Plain definitions used to pin the simulation
+# ---------------------------------------------------------------------------
+
+def column_reduce_exact(inputs, op: str, dtype: str):
+    """The Allreduce result from its definition, u_{i,Sigma} = u_{i,0} (+) ... (+)
+    u_{i,P-1} (Sec. "Combination of distributed data vectors"), for the cases where it
+    has a unique value: i32 sum in exact integers reduced mod 2^32 (two's complement),
+    and max/min of any type."""
+    stack = np.stack([np.asarray(v) for v in inputs])
+    if op == "sum":
+        if dtype != "i32":
+            raise ValueError("floating-point sums depend on association order")
+        tot = stack.astype(np.int64).sum(axis=0)          # exact for P < 2^32
+        wrapped = ((tot + 2**31) % 2**32) - 2**31
+        return wrapped.astype(np.int32)
+    if op == "max":
+        return stack.max(axis=0)
+    if op == "min":
+        return stack.min(axis=0)
+    raise ValueError(op)
+
+
+def kahan_sum_f64(inputs) -> tuple[np.ndarray, np.ndarray]:
+    """Compensated (Kahan) sum of the P inputs in rank order, in float64, and the sum
+    of absolute values (the scale of the standard summation error bound)."""
+    stack = np.stack([np.asarray(v, dtype=np.float64) for v in inputs])
+    s = np.zeros(stack.shape[1], dtype=np.float64)
+    comp = np.zeros_like(s)
+    for row in stack:
+        y = row - comp
+        t = s + y
+        comp = (t - s) - y
+        s = t
+    return s, np.abs(stack).sum(axis=0)
+
+
+# ---------------------------------------------------------------------------
+# Cost model (Sec. "Communication model"; eqs. bo_cost, intemediate_cost, lo_cost)
+# ---------------------------------------------------------------------------
+
+def cost_model_time(P: int, m_bytes: float, steps: int, alpha: float, beta: float,
+                    gamma: float) -> float:
+    """tau for the version with S = steps (eq. bo_cost for r = 0, eq. intemediate_cost
+    for 0 < r < L, eq. lo_cost for r = L), with u = m/P."""
+    L = ceil_log2(P)
+    r = 2 * L - steps
+    if not 0 <= r <= L:
+        raise ValueError("steps out of range")
+    u = m_bytes / P
+    if r == L:
+        return L * alpha + P * L * u * beta + P * (2 * L - 2) * u * gamma
+    return ((2 * L - r) * alpha
+            + (2 * (P - 1) + (2 ** r - 1) * (L - 1)) * u * beta
+            + ((P - 1) + (2 ** r - 1) * (2 * L - 2)) * u * gamma)
+
+
+def optimal_steps(P: int, m_bytes: float, alpha: float, beta: float, gamma: float) -> int:
+    """The step count minimising the cost model over integer S in [L, 2L] (eq.
+    opt_number_of_steps gives the continuous optimum; reading C15 takes the argmin)."""
+    L = ceil_log2(P)
+    if L == 0:
+        return 0
+    best = None
+    for S in range(L, 2 * L + 1):
+        t = cost_model_time(P, m_bytes, S, alpha, beta, gamma)
+        if best is None or t < best[0] - 1e-18:
+            best = (t, S)
+    return best[1]
