@@ -1,0 +1,213 @@
+/*
+ * gar.h -- permutation-group Allreduce on one GB300 (sm_103a).
+ *
+ * Implements the generalized Allreduce of D. Kolmakov and X. Zhang, "A Generalization
+ * of the Allreduce Operation" (arXiv 2004.09362): the schedule built from the cyclic
+ * permutation group T_P, with a step count S that can be set anywhere from
+ * ceil(log2 P) (latency-optimal, Sec. "Latency-optimal version") to 2 ceil(log2 P)
+ * (bandwidth-optimal, Sec. "Bandwidth-optimal algorithm") for any P, including
+ * non-powers of two and primes (Sec. "Moving towards latency-optimal version").
+ *
+ * The P processes of the paper are P "virtual ranks": P equally sized vectors that
+ * all live in the memory of one GPU.  A message of the paper is a read of the partner
+ * rank's block.  Semantics follow MPI_Allreduce with MPI_IN_PLACE (Sec.
+ * "Introduction"): after the call every rank buffer holds the op-reduction of all P
+ * input vectors.
+ *
+ * Conventions for every function below:
+ *  - Return value: GAR_OK (0) on success, a negative GAR_E* code otherwise.  No error
+ *    is raised asynchronously by the library itself; a CUDA error from an earlier
+ *    kernel surfaces as GAR_ECUDA from the next call that checks.  gar_strerror()
+ *    names a code; gar_last_error() gives the calling thread's last detail message.
+ *  - Ownership: rank buffers, workspaces and batch descriptor arrays belong to the
+ *    caller.  A plan owns its host tables and the small device tables it uploads
+ *    (descriptors, byte counters); gar_plan_destroy frees them.
+ *  - Ordering: functions taking a stream enqueue work on it and return without
+ *    waiting, except where stated.  A plan may be used from one host thread at a time.
+ *  - Device pointers must point into memory of the current CUDA device.
+ */
+#ifndef GAR_H
+#define GAR_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#if defined(__GNUC__)
+#define GAR_API __attribute__((visibility("default")))
+#else
+#define GAR_API
+#endif
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef struct gar_plan gar_plan;
+typedef struct CUstream_st *gar_stream_t; /* identical to cudaStream_t */
+
+/* Element types.  GAR_BF16 combines in fp32 and rounds once to bf16 (round to
+ * nearest even) when a result is written. */
+enum { GAR_F32 = 0, GAR_BF16 = 1, GAR_I32 = 2 };
+
+/* Reduction operators.  Only commutative operators: the method reorders operands
+ * (Sec. "Related work" names commutativity as the condition for cyclic patterns).
+ * GAR_SUM on GAR_I32 wraps modulo 2^32. */
+enum { GAR_SUM = 0, GAR_MAX = 1, GAR_MIN = 2 };
+
+/* Execution modes.
+ * GAR_STEP_FAITHFUL: one kernel launch per schedule step; a step reads the
+ *   partner rank's blocks (the paper's send/receive) with 16-byte vector loads and
+ *   combines them with the own block; needs the workspace reported by
+ *   gar_plan_bytes; records the bytes read from partners per step.
+ * GAR_FUSED: one launch for the whole Allreduce; per element position the P
+ *   contributions are loaded once, the reduction program that the schedule induces
+ *   runs in registers, and every rank's result is written once. */
+enum { GAR_STEP_FAITHFUL = 0, GAR_FUSED = 1 };
+
+/* Special values for the `steps` argument of gar_plan_create. */
+#define GAR_STEPS_BO (-1) /* 2 ceil(log2 P): bandwidth-optimal */
+#define GAR_STEPS_LO (-2) /* ceil(log2 P): latency-optimal */
+
+#define GAR_MAX_P 1024 /* largest supported number of virtual ranks */
+
+enum {
+  GAR_OK = 0,
+  GAR_EINVAL = -1,  /* bad argument (P, n, dtype, op, steps, mode, null pointer) */
+  GAR_ENOMEM = -2,  /* host or device allocation failed */
+  GAR_EALIGN = -3,  /* a buffer is not 16-byte aligned */
+  GAR_ECUDA = -4,   /* a CUDA runtime call failed (detail in gar_last_error) */
+  GAR_EJIT = -5,    /* run-time compilation of a specialized kernel failed */
+  GAR_ENOWS = -6,   /* step-faithful mode needs a workspace that was not set or is too small */
+  GAR_ESTATE = -7   /* operation not valid in the plan's current state */
+};
+
+/* Describes a plan.  Symbols follow the paper: L = ceil(log2 P) reduction steps
+ * (eq. bo_starting_set_size), S = 2L - r total steps, K = number of q_Sigma copies at
+ * the end of the reduction phase (K = N_{L-r}; K = 1 bandwidth-optimal, K = P
+ * latency-optimal). */
+typedef struct {
+  int32_t P;
+  int32_t L;
+  int32_t S;
+  int32_t r;
+  int32_t K;
+  int32_t dtype;
+  int32_t op;
+  int32_t n_launches;        /* step-faithful kernel launches per Allreduce */
+  uint64_t n;                /* elements per rank */
+  int32_t fused_combines;    /* combines per element position in fused mode */
+  int32_t fused_width;       /* elements per thread-vector in the fused kernel */
+} gar_plan_info;
+
+/* Creates a schedule for P virtual ranks of n elements each.
+ * P: 1..GAR_MAX_P.  n: elements per rank (0 is allowed: every call is a no-op).
+ * steps: S in [ceil(log2 P), 2 ceil(log2 P)], or GAR_STEPS_BO / GAR_STEPS_LO.
+ * The block partition is the paper's V_j = (u_{0,j}, ..., u_{P-1,j}) (eq.
+ * initial_data) with the first n mod P blocks one element longer.  Host-only: needs
+ * no GPU.  *out is set only on success. */
+GAR_API int gar_plan_create(gar_plan **out, int P, uint64_t n, int dtype, int op, int steps);
+
+/* Frees the plan and its device tables.  NULL is a no-op.  The caller must make sure
+ * no work using the plan is still running. */
+GAR_API void gar_plan_destroy(gar_plan *plan);
+
+GAR_API int gar_plan_get_info(const gar_plan *plan, gar_plan_info *info);
+
+/* Sizes.  workspace_bytes: device workspace step-faithful mode needs (0 when the
+ * schedule runs in place: bandwidth-optimal f32/i32).  msg_bytes_per_step (may be
+ * NULL, else S entries): bytes all ranks together read from their partners in each
+ * communication step, the schedule's message volume (Sec. "Communication
+ * operator": every rank sends its blocks of the transmitted vectors).  S (may be
+ * NULL) receives the step count.  Host-only. */
+GAR_API int gar_plan_bytes(const gar_plan *plan, size_t *workspace_bytes,
+                   uint64_t *msg_bytes_per_step, int *S);
+
+/* Schedule introspection (host-only).  For communication step t in [0, S):
+ * phase = 0 (reduction) or 1 (distribution); partner = offset so that rank x
+ * receives from rank (x + partner) mod P (reduction: +floor(N_i/2), eq. bo_dir_perms;
+ * distribution: -floor(N_i/2)); placements[0..*count) = placements of the vectors
+ * each rank transmits (eq. bo_tx_dist and its shifted forms).  placements may be
+ * NULL to query the count; otherwise it must hold P entries. */
+GAR_API int gar_plan_step(const gar_plan *plan, int t, int *phase, int *partner,
+                  int32_t *placements, int *count);
+
+/* origin[p] for p in [0, P): the result copy (0..K-1) that placement p receives in the
+ * distribution phase.  Rank x's result for block b is placement (x - b) mod P. */
+GAR_API int gar_plan_origin(const gar_plan *plan, int32_t *origin);
+
+/* The fused-mode program: value ids 0..P-1 are the P contributions of an element
+ * position rotated by its block b (id j = rank (b + j) mod P); combine k makes value
+ * P + k = ops[2k] (+) ops[2k+1] (own, received).  outputs[s] (s < K) = value id of
+ * result copy s.  Pass NULL arrays to query *nops; ops must hold 2 * *nops entries and
+ * outputs K entries. */
+GAR_API int gar_plan_fused_program(const gar_plan *plan, int32_t *ops, int *nops, int32_t *outputs);
+
+/* The step-faithful op table (host-only, for inspection and tests).  Each op is 8
+ * int32: {launch, recv_place, dst_place, recv_buf, out0_buf, out0_own, out1_buf,
+ * out1_own}; buffers: 0 none, 1 rank buffer, 2 q' ping, 3 q' pong, 4 q* store.
+ * launch_partner[l] = receive offset of launch l.  Query *nops with ops == NULL. */
+GAR_API int gar_plan_step_ops(const gar_plan *plan, int32_t *ops, int *nops, int32_t *launch_partner,
+                      int *nlaunch);
+
+/* Caller-owned device workspace for step-faithful mode (16-byte aligned, at least
+ * workspace_bytes).  NULL with 0 bytes detaches it. */
+GAR_API int gar_plan_set_workspace(gar_plan *plan, void *dev_ptr, size_t bytes);
+
+/* Compiles (host-only, needs no GPU) the specialized kernel for `mode`.  Optional:
+ * gar_plan_prepare and the first Allreduce compile on demand. */
+GAR_API int gar_plan_compile(gar_plan *plan, int mode);
+
+/* Compiles and loads everything `mode` needs on the current device and uploads the
+ * device tables.  Call before capturing Allreduce calls into a CUDA graph. */
+GAR_API int gar_plan_prepare(gar_plan *plan, int mode);
+
+/* The Allreduce (MPI_Allreduce with MPI_IN_PLACE, Sec. "Introduction").
+ * rank_buffers: host array of P device pointers, each to n elements of the plan's
+ * type, 16-byte aligned and pairwise distinct.  On return the work is enqueued on
+ * `stream`; when it completes every buffer holds the reduction.  Rank x's block b is
+ * the value at placement (x - b) mod P after the paper's schedule; for bandwidth-
+ * optimal plans all ranks get identical bits, otherwise floating-point sums may differ
+ * in the last bits between ranks (each rank's association order is a rotation of the
+ * same tree). */
+GAR_API int gar_allreduce(gar_plan *plan, void *const *rank_buffers, int mode, gar_stream_t stream);
+
+/* Host-buffer Allreduce: copies host_in[x] (P host pointers, pinned memory gives full
+ * speed) to dev_bufs[x], runs gar_allreduce on dev_bufs, and copies the results to
+ * host_out[x] (may equal host_in).  Each copy is one cudaMemcpyAsync on `stream`.
+ * Returns after enqueueing; synchronize the stream before reading host_out. */
+GAR_API int gar_allreduce_host(gar_plan *plan, const void *const *host_in, void *const *host_out,
+                       void *const *dev_bufs, int mode, gar_stream_t stream);
+
+/* One instance of a batched Allreduce: `in` and `out` point to row-major [P][n]
+ * arrays (rank x's vector is row x) for plans[plan]; in == out is allowed. */
+typedef struct {
+  int32_t plan;
+  int32_t reserved;
+  const void *in;
+  void *out;
+} gar_batch_desc;
+
+/* Many independent small Allreduces in one fused launch (the 425-byte Allreduce of
+ * Sec. "Introduction").  plans: nplans plans sharing dtype, op and n.  desc: DEVICE
+ * array of `count` descriptors.  Instances whose pointers are not aligned for the
+ * kernel's vector width fall back to element-wise loads inside the same kernel. */
+GAR_API int gar_allreduce_batched(gar_plan *const *plans, int nplans, const gar_batch_desc *desc,
+                          int count, gar_stream_t stream);
+
+/* Bytes each communication step of the most recent step-faithful Allreduce read from
+ * partner ranks, as counted by the kernels (S entries).  Synchronizes with the stream
+ * of that call. */
+GAR_API int gar_last_step_bytes(const gar_plan *plan, uint64_t *per_step);
+
+GAR_API const char *gar_strerror(int status);
+GAR_API const char *gar_last_error(void);
+
+/* Library self-test for build checks: generates and compiles (host-only, no GPU) the
+ * fused kernels of a few plans.  Returns GAR_OK or GAR_EJIT. */
+GAR_API int gar_selftest_compile(void);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* GAR_H */

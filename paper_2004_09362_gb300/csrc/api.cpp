@@ -1,0 +1,472 @@
+// C ABI of the permutation-group Allreduce library (declared in include/gar.h).
+#include <cuda_runtime.h>
+
+#include <algorithm>
+#include <cstring>
+#include <new>
+#include <string>
+#include <vector>
+
+#include "gar_internal.hpp"
+
+namespace gar {
+
+namespace {
+thread_local std::string t_last_error;
+}
+
+void set_error(const std::string &msg) { t_last_error = msg; }
+const char *last_error_cstr() { return t_last_error.c_str(); }
+
+int cuda_fail(int err, const char *what) {
+  set_error(std::string(what) + ": " + cudaGetErrorString((cudaError_t)err));
+  return GAR_ECUDA;
+}
+
+namespace {
+
+int check_plan(const gar_plan *pl) {
+  if (pl == nullptr) {
+    set_error("null plan");
+    return GAR_EINVAL;
+  }
+  return GAR_OK;
+}
+
+int check_mode(int mode) {
+  if (mode != GAR_STEP_FAITHFUL && mode != GAR_FUSED) {
+    set_error("unknown mode");
+    return GAR_EINVAL;
+  }
+  return GAR_OK;
+}
+
+int ensure_device(gar_plan *pl) {
+  int dev = -1;
+  cudaError_t e = cudaGetDevice(&dev);
+  if (e != cudaSuccess) return cuda_fail(e, "cudaGetDevice");
+  if (pl->device >= 0 && pl->device != dev) {
+    set_error("plan was prepared on another device");
+    return GAR_ESTATE;
+  }
+  pl->device = dev;
+  return GAR_OK;
+}
+
+int prepare_step_faithful(gar_plan *pl) {
+  int rc = ensure_device(pl);
+  if (rc) return rc;
+  if (pl->d_ops == nullptr && !pl->ops.empty()) {
+    cudaError_t e = cudaMalloc(&pl->d_ops, pl->ops.size() * sizeof(StepOp));
+    if (e != cudaSuccess) return cuda_fail(e, "cudaMalloc(op table)");
+    e = cudaMemcpy(pl->d_ops, pl->ops.data(), pl->ops.size() * sizeof(StepOp),
+                   cudaMemcpyHostToDevice);
+    if (e != cudaSuccess) return cuda_fail(e, "cudaMemcpy(op table)");
+  }
+  if (pl->d_step_bytes == nullptr && pl->S > 0) {
+    cudaError_t e = cudaMalloc(&pl->d_step_bytes, pl->S * sizeof(unsigned long long));
+    if (e != cudaSuccess) return cuda_fail(e, "cudaMalloc(step counters)");
+    e = cudaMemset(pl->d_step_bytes, 0, pl->S * sizeof(unsigned long long));
+    if (e != cudaSuccess) return cuda_fail(e, "cudaMemset(step counters)");
+  }
+  return GAR_OK;
+}
+
+int compile_fused(gar_plan *pl) {
+  if (pl->fused) return GAR_OK;
+  CodegenResult cg = generate_fused_source(*pl);
+  JitKernel *k = nullptr;
+  int rc = jit_compile(cg, &k);
+  if (rc) return rc;
+  pl->fused = k;
+  pl->fused_width = k->width;
+  return GAR_OK;
+}
+
+int prepare_fused(gar_plan *pl) {
+  int rc = compile_fused(pl);
+  if (rc) return rc;
+  rc = ensure_device(pl);
+  if (rc) return rc;
+  return jit_load(pl->fused);
+}
+
+int check_buffers(const gar_plan *pl, void *const *bufs) {
+  if (bufs == nullptr) {
+    set_error("null rank buffer array");
+    return GAR_EINVAL;
+  }
+  std::vector<uintptr_t> ptrs(pl->P);
+  for (int x = 0; x < pl->P; ++x) {
+    if (bufs[x] == nullptr) {
+      set_error("null rank buffer " + std::to_string(x));
+      return GAR_EINVAL;
+    }
+    if (reinterpret_cast<uintptr_t>(bufs[x]) % 16 != 0) {
+      set_error("rank buffer " + std::to_string(x) + " is not 16-byte aligned");
+      return GAR_EALIGN;
+    }
+    ptrs[x] = reinterpret_cast<uintptr_t>(bufs[x]);
+  }
+  std::sort(ptrs.begin(), ptrs.end());
+  if (std::adjacent_find(ptrs.begin(), ptrs.end()) != ptrs.end()) {
+    set_error("two ranks share one buffer");
+    return GAR_EINVAL;
+  }
+  return GAR_OK;
+}
+
+int grid_for(const JitKernel *k, uint64_t work_items) {
+  int dev = 0, sms = 0;
+  cudaGetDevice(&dev);
+  cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
+  if (sms <= 0) sms = 1;
+  const uint64_t need = (work_items + k->threads - 1) / k->threads;
+  const uint64_t wave = (uint64_t)sms * (uint64_t)std::max(1, k->blocks_per_sm);
+  return (int)std::max<uint64_t>(1, std::min<uint64_t>(need, wave));
+}
+
+int run_fused(gar_plan *pl, void *const *rank, gar_stream_t stream) {
+  int rc = prepare_fused(pl);
+  if (rc) return rc;
+  std::vector<void *> args(rank, rank + pl->P);
+  void *kargs[] = {args.data()};
+  const uint64_t items = pl->n / pl->fused->width + 1;
+  const int grid = grid_for(pl->fused, items);
+  cudaError_t e = cudaLaunchKernel((const void *)pl->fused->kernel, dim3(grid),
+                                   dim3(pl->fused->threads), kargs, 0, (cudaStream_t)stream);
+  if (e != cudaSuccess) return cuda_fail(e, "fused kernel launch");
+  return GAR_OK;
+}
+
+int run_step_faithful(gar_plan *pl, void *const *rank, gar_stream_t stream) {
+  int rc = prepare_step_faithful(pl);
+  if (rc) return rc;
+  if (pl->ws_bytes > 0) {
+    if (pl->ws == nullptr || pl->ws_set_bytes < pl->ws_bytes) {
+      set_error("step-faithful mode needs a workspace of " + std::to_string(pl->ws_bytes) +
+                " bytes (gar_plan_set_workspace)");
+      return GAR_ENOWS;
+    }
+  }
+  cudaError_t e = cudaMemsetAsync(pl->d_step_bytes, 0, pl->S * sizeof(unsigned long long),
+                                  (cudaStream_t)stream);
+  if (e != cudaSuccess) return cuda_fail(e, "cudaMemsetAsync(step counters)");
+  for (size_t li = 0; li < pl->launches.size(); ++li) {
+    rc = launch_step(*pl, pl->launches[li], (int)li, rank, stream);
+    if (rc) return rc;
+  }
+  pl->last_stream = stream;
+  pl->ran_step_faithful = true;
+  return GAR_OK;
+}
+
+}  // namespace
+}  // namespace gar
+
+using namespace gar;
+
+extern "C" {
+
+int gar_plan_create(gar_plan **out, int P, uint64_t n, int dtype, int op, int steps) {
+  if (out == nullptr) {
+    set_error("null output pointer");
+    return GAR_EINVAL;
+  }
+  if (P < 1 || P > GAR_MAX_P) {
+    set_error("P must be in [1, " + std::to_string(GAR_MAX_P) + "]");
+    return GAR_EINVAL;
+  }
+  if (dtype != GAR_F32 && dtype != GAR_BF16 && dtype != GAR_I32) {
+    set_error("unknown dtype");
+    return GAR_EINVAL;
+  }
+  if (op != GAR_SUM && op != GAR_MAX && op != GAR_MIN) {
+    set_error("unknown op");
+    return GAR_EINVAL;
+  }
+  if (n > (uint64_t)1 << 40) {
+    set_error("n too large");
+    return GAR_EINVAL;
+  }
+  const int L = ceil_log2(P);
+  int S = steps;
+  if (steps == GAR_STEPS_BO) S = 2 * L;
+  if (steps == GAR_STEPS_LO) S = L;
+  if (S < L || S > 2 * L) {
+    set_error("steps must be in [" + std::to_string(L) + ", " + std::to_string(2 * L) + "] for P=" +
+              std::to_string(P));
+    return GAR_EINVAL;
+  }
+  gar_plan *pl = new (std::nothrow) gar_plan();
+  if (pl == nullptr) return GAR_ENOMEM;
+  pl->P = P;
+  pl->n = n;
+  pl->dtype = dtype;
+  pl->op = op;
+  pl->S = S;
+  int rc = build_plan(pl);
+  if (rc) {
+    delete pl;
+    return rc;
+  }
+  *out = pl;
+  return GAR_OK;
+}
+
+void gar_plan_destroy(gar_plan *pl) {
+  if (pl == nullptr) return;
+  if (pl->d_ops) cudaFree(pl->d_ops);
+  if (pl->d_step_bytes) cudaFree(pl->d_step_bytes);
+  delete pl;
+}
+
+int gar_plan_get_info(const gar_plan *pl, gar_plan_info *info) {
+  if (int rc = check_plan(pl)) return rc;
+  if (info == nullptr) return GAR_EINVAL;
+  std::memset(info, 0, sizeof *info);
+  info->P = pl->P;
+  info->L = pl->L;
+  info->S = pl->S;
+  info->r = pl->r;
+  info->K = pl->K;
+  info->dtype = pl->dtype;
+  info->op = pl->op;
+  info->n_launches = (int)pl->launches.size();
+  info->n = pl->n;
+  info->fused_combines = (int)pl->prog.a.size();
+  info->fused_width = pl->fused_width;
+  return GAR_OK;
+}
+
+int gar_plan_bytes(const gar_plan *pl, size_t *workspace_bytes, uint64_t *msg_bytes_per_step, int *S) {
+  if (int rc = check_plan(pl)) return rc;
+  if (workspace_bytes) *workspace_bytes = pl->ws_bytes;
+  if (msg_bytes_per_step)
+    for (int t = 0; t < pl->S; ++t) msg_bytes_per_step[t] = pl->comm[t].msg_bytes;
+  if (S) *S = pl->S;
+  return GAR_OK;
+}
+
+int gar_plan_step(const gar_plan *pl, int t, int *phase, int *partner, int32_t *placements, int *count) {
+  if (int rc = check_plan(pl)) return rc;
+  if (t < 0 || t >= pl->S) {
+    set_error("step index out of range");
+    return GAR_EINVAL;
+  }
+  const CommStep &cs = pl->comm[t];
+  if (phase) *phase = cs.phase;
+  if (partner) *partner = cs.partner;
+  if (count) *count = (int)cs.tx.size();
+  if (placements) std::copy(cs.tx.begin(), cs.tx.end(), placements);
+  return GAR_OK;
+}
+
+int gar_plan_origin(const gar_plan *pl, int32_t *origin) {
+  if (int rc = check_plan(pl)) return rc;
+  if (origin == nullptr) return GAR_EINVAL;
+  std::copy(pl->prog.origin.begin(), pl->prog.origin.end(), origin);
+  return GAR_OK;
+}
+
+int gar_plan_fused_program(const gar_plan *pl, int32_t *ops, int *nops, int32_t *outputs) {
+  if (int rc = check_plan(pl)) return rc;
+  if (nops == nullptr) return GAR_EINVAL;
+  *nops = (int)pl->prog.a.size();
+  if (ops)
+    for (size_t k = 0; k < pl->prog.a.size(); ++k) {
+      ops[2 * k] = pl->prog.a[k];
+      ops[2 * k + 1] = pl->prog.b[k];
+    }
+  if (outputs) std::copy(pl->prog.out.begin(), pl->prog.out.end(), outputs);
+  return GAR_OK;
+}
+
+int gar_plan_step_ops(const gar_plan *pl, int32_t *ops, int *nops, int32_t *launch_partner, int *nlaunch) {
+  if (int rc = check_plan(pl)) return rc;
+  if (nops) *nops = (int)pl->ops.size();
+  if (nlaunch) *nlaunch = (int)pl->launches.size();
+  if (launch_partner)
+    for (size_t l = 0; l < pl->launches.size(); ++l) launch_partner[l] = pl->launches[l].partner;
+  if (ops) {
+    for (size_t l = 0; l < pl->launches.size(); ++l) {
+      const Launch &ln = pl->launches[l];
+      for (int k = 0; k < ln.nops; ++k) {
+        const StepOp &op = pl->ops[ln.first_op + k];
+        int32_t *o = ops + 8 * (size_t)(ln.first_op + k);
+        o[0] = (int32_t)l;
+        o[1] = op.recv_place;
+        o[2] = op.dst_place;
+        o[3] = op.recv_buf;
+        o[4] = op.out0_buf;
+        o[5] = op.out0_own;
+        o[6] = op.out1_buf;
+        o[7] = op.out1_own;
+      }
+    }
+  }
+  return GAR_OK;
+}
+
+int gar_plan_set_workspace(gar_plan *pl, void *dev_ptr, size_t bytes) {
+  if (int rc = check_plan(pl)) return rc;
+  if (dev_ptr == nullptr && bytes != 0) return GAR_EINVAL;
+  if (reinterpret_cast<uintptr_t>(dev_ptr) % 16 != 0) {
+    set_error("workspace is not 16-byte aligned");
+    return GAR_EALIGN;
+  }
+  pl->ws = dev_ptr;
+  pl->ws_set_bytes = bytes;
+  return GAR_OK;
+}
+
+int gar_plan_compile(gar_plan *pl, int mode) {
+  if (int rc = check_plan(pl)) return rc;
+  if (int rc = check_mode(mode)) return rc;
+  if (mode == GAR_FUSED) return compile_fused(pl);
+  return GAR_OK;
+}
+
+int gar_plan_prepare(gar_plan *pl, int mode) {
+  if (int rc = check_plan(pl)) return rc;
+  if (int rc = check_mode(mode)) return rc;
+  if (mode == GAR_FUSED) return prepare_fused(pl);
+  return prepare_step_faithful(pl);
+}
+
+int gar_allreduce(gar_plan *pl, void *const *rank_buffers, int mode, gar_stream_t stream) {
+  if (int rc = check_plan(pl)) return rc;
+  if (int rc = check_mode(mode)) return rc;
+  if (int rc = check_buffers(pl, rank_buffers)) return rc;
+  if (pl->n == 0 || pl->P == 1) return GAR_OK;
+  return mode == GAR_FUSED ? run_fused(pl, rank_buffers, stream)
+                           : run_step_faithful(pl, rank_buffers, stream);
+}
+
+int gar_allreduce_host(gar_plan *pl, const void *const *host_in, void *const *host_out,
+                       void *const *dev_bufs, int mode, gar_stream_t stream) {
+  if (int rc = check_plan(pl)) return rc;
+  if (int rc = check_mode(mode)) return rc;
+  if (host_in == nullptr || host_out == nullptr) {
+    set_error("null host buffer array");
+    return GAR_EINVAL;
+  }
+  if (int rc = check_buffers(pl, dev_bufs)) return rc;
+  const size_t bytes = (size_t)pl->n * (size_t)elem_size(pl->dtype);
+  for (int x = 0; x < pl->P; ++x) {
+    if (host_in[x] == nullptr || host_out[x] == nullptr) {
+      set_error("null host buffer");
+      return GAR_EINVAL;
+    }
+  }
+  for (int x = 0; x < pl->P && bytes; ++x) {
+    cudaError_t e = cudaMemcpyAsync(dev_bufs[x], host_in[x], bytes, cudaMemcpyHostToDevice,
+                                    (cudaStream_t)stream);
+    if (e != cudaSuccess) return cuda_fail(e, "cudaMemcpyAsync(host to device)");
+  }
+  int rc = gar_allreduce(pl, dev_bufs, mode, stream);
+  if (rc) return rc;
+  for (int x = 0; x < pl->P && bytes; ++x) {
+    cudaError_t e = cudaMemcpyAsync(host_out[x], dev_bufs[x], bytes, cudaMemcpyDeviceToHost,
+                                    (cudaStream_t)stream);
+    if (e != cudaSuccess) return cuda_fail(e, "cudaMemcpyAsync(device to host)");
+  }
+  return GAR_OK;
+}
+
+int gar_allreduce_batched(gar_plan *const *plans, int nplans, const gar_batch_desc *desc, int count,
+                          gar_stream_t stream) {
+  if (plans == nullptr || nplans < 1 || count < 0 || (count > 0 && desc == nullptr)) {
+    set_error("bad batched arguments");
+    return GAR_EINVAL;
+  }
+  std::vector<const gar_plan *> ps;
+  for (int k = 0; k < nplans; ++k) {
+    if (plans[k] == nullptr) {
+      set_error("null plan in batch");
+      return GAR_EINVAL;
+    }
+    if (plans[k]->dtype != plans[0]->dtype || plans[k]->op != plans[0]->op ||
+        plans[k]->n != plans[0]->n) {
+      set_error("batched plans must share dtype, op and n");
+      return GAR_EINVAL;
+    }
+    ps.push_back(plans[k]);
+  }
+  if (count == 0 || plans[0]->n == 0) return GAR_OK;
+  if (reinterpret_cast<uintptr_t>(desc) % 8 != 0) {
+    set_error("descriptor array is not 8-byte aligned");
+    return GAR_EALIGN;
+  }
+  CodegenResult cg = generate_batched_source(ps);
+  JitKernel *k = nullptr;
+  int rc = jit_compile(cg, &k);
+  if (rc) return rc;
+  rc = jit_load(k);
+  if (rc) return rc;
+  struct {
+    const gar_batch_desc *desc;
+    unsigned long long count;
+  } a = {desc, (unsigned long long)count};
+  void *kargs[] = {&a};
+  const uint64_t per = plans[0]->n / k->width + plans[0]->n % k->width;
+  const int grid = grid_for(k, per * (uint64_t)count);
+  cudaError_t e = cudaLaunchKernel((const void *)k->kernel, dim3(grid), dim3(k->threads), kargs, 0,
+                                   (cudaStream_t)stream);
+  if (e != cudaSuccess) return cuda_fail(e, "batched kernel launch");
+  return GAR_OK;
+}
+
+int gar_last_step_bytes(const gar_plan *pl, uint64_t *per_step) {
+  if (int rc = check_plan(pl)) return rc;
+  if (per_step == nullptr) return GAR_EINVAL;
+  if (!pl->ran_step_faithful) {
+    set_error("no step-faithful Allreduce has run on this plan");
+    return GAR_ESTATE;
+  }
+  cudaError_t e = cudaStreamSynchronize((cudaStream_t)pl->last_stream);
+  if (e != cudaSuccess) return cuda_fail(e, "cudaStreamSynchronize");
+  std::vector<unsigned long long> tmp(pl->S);
+  e = cudaMemcpy(tmp.data(), pl->d_step_bytes, pl->S * sizeof(unsigned long long),
+                 cudaMemcpyDeviceToHost);
+  if (e != cudaSuccess) return cuda_fail(e, "cudaMemcpy(step counters)");
+  for (int t = 0; t < pl->S; ++t) per_step[t] = tmp[t];
+  return GAR_OK;
+}
+
+const char *gar_strerror(int status) {
+  switch (status) {
+    case GAR_OK: return "success";
+    case GAR_EINVAL: return "invalid argument";
+    case GAR_ENOMEM: return "out of memory";
+    case GAR_EALIGN: return "buffer not 16-byte aligned";
+    case GAR_ECUDA: return "CUDA error";
+    case GAR_EJIT: return "kernel compilation failed";
+    case GAR_ENOWS: return "workspace missing or too small";
+    case GAR_ESTATE: return "invalid plan state";
+  }
+  return "unknown status";
+}
+
+const char *gar_last_error(void) { return last_error_cstr(); }
+
+int gar_selftest_compile(void) {
+  const int cases[][4] = {{24, GAR_F32, GAR_SUM, -1}, {7, GAR_F32, GAR_MAX, 3},
+                          {5, GAR_BF16, GAR_SUM, 4},  {6, GAR_I32, GAR_MIN, 3}};
+  for (const auto &c : cases) {
+    gar_plan *pl = nullptr;
+    int rc = gar_plan_create(&pl, c[0], 1000 + c[0], c[1], c[2], c[3]);
+    if (rc) return rc;
+    rc = gar_plan_compile(pl, GAR_FUSED);
+    if (rc == GAR_OK) {
+      std::vector<const gar_plan *> ps{pl};
+      JitKernel *k = nullptr;
+      rc = jit_compile(generate_batched_source(ps), &k);
+    }
+    gar_plan_destroy(pl);
+    if (rc) return rc;
+  }
+  return GAR_OK;
+}
+
+}  // extern "C"

@@ -1,0 +1,413 @@
+// Code generator for the fused and batched kernels.
+//
+// A plan's fused program (plan.cpp) is a short straight-line list of combines per
+// element position.  Emitting it as straight-line CUDA C and compiling it for sm_103a
+// at plan creation (jit.cpp) keeps every contribution and partial result in registers
+// with compile-time indices, for any P and any step count, instead of interpreting the
+// schedule from a table at run time.  The fixed parts of the kernels (vector loads
+// and stores, bf16 handling, grid-stride loops) are the text in kSkeleton below.
+#include <algorithm>
+#include <cstdarg>
+#include <cstdio>
+#include <functional>
+#include <string>
+#include <vector>
+
+#include "gar_internal.hpp"
+
+namespace gar {
+namespace {
+
+// Types, operators and 1..16-byte vector loads/stores shared by every generated kernel.
+// Loads and stores use the streaming cache hints (.cs): every byte is touched once.
+const char *kSkeleton = R"CUDA(
+typedef unsigned short gar_u16;
+typedef unsigned int gar_u32;
+typedef unsigned long long gar_u64;
+
+#if GAR_DTYPE == 1
+typedef float gar_acc;
+typedef gar_u16 gar_io;
+#elif GAR_DTYPE == 2
+typedef int gar_acc;
+typedef int gar_io;
+#else
+typedef float gar_acc;
+typedef float gar_io;
+#endif
+
+static __device__ __forceinline__ gar_acc gar_op(gar_acc a, gar_acc b) {
+#if GAR_DTYPE == 2
+#if GAR_OP == 0
+  return (int)((gar_u32)a + (gar_u32)b);
+#elif GAR_OP == 1
+  return a > b ? a : b;
+#else
+  return a < b ? a : b;
+#endif
+#else
+#if GAR_OP == 0
+  return a + b;
+#elif GAR_OP == 1
+  return fmaxf(a, b);
+#else
+  return fminf(a, b);
+#endif
+#endif
+}
+
+static __device__ __forceinline__ float gar_bf16_lo(gar_u32 u) { return __uint_as_float(u << 16); }
+static __device__ __forceinline__ float gar_bf16_hi(gar_u32 u) { return __uint_as_float(u & 0xffff0000u); }
+static __device__ __forceinline__ gar_u32 gar_pack_bf16(float lo, float hi) {
+  gar_u32 r;
+  asm("cvt.rn.bf16x2.f32 %0, %1, %2;" : "=r"(r) : "f"(hi), "f"(lo));
+  return r;
+}
+
+// Load W consecutive elements at p (aligned to W elements) into v[0..W).
+template <int W> static __device__ __forceinline__ void gar_load(const gar_io *p, gar_acc *v);
+template <int W> static __device__ __forceinline__ void gar_store(gar_io *p, const gar_acc *v);
+
+#if GAR_DTYPE == 1
+template <> __device__ __forceinline__ void gar_load<1>(const gar_io *p, gar_acc *v) {
+  gar_u16 h;
+  asm("ld.global.cs.u16 %0, [%1];" : "=h"(h) : "l"(p));
+  v[0] = __uint_as_float(((gar_u32)h) << 16);
+}
+template <> __device__ __forceinline__ void gar_load<2>(const gar_io *p, gar_acc *v) {
+  gar_u32 u;
+  asm("ld.global.cs.u32 %0, [%1];" : "=r"(u) : "l"(p));
+  v[0] = gar_bf16_lo(u); v[1] = gar_bf16_hi(u);
+}
+template <> __device__ __forceinline__ void gar_load<4>(const gar_io *p, gar_acc *v) {
+  gar_u32 a, b;
+  asm("ld.global.cs.v2.u32 {%0,%1}, [%2];" : "=r"(a), "=r"(b) : "l"(p));
+  v[0] = gar_bf16_lo(a); v[1] = gar_bf16_hi(a); v[2] = gar_bf16_lo(b); v[3] = gar_bf16_hi(b);
+}
+template <> __device__ __forceinline__ void gar_load<8>(const gar_io *p, gar_acc *v) {
+  gar_u32 a, b, c, d;
+  asm("ld.global.cs.v4.u32 {%0,%1,%2,%3}, [%4];" : "=r"(a), "=r"(b), "=r"(c), "=r"(d) : "l"(p));
+  v[0] = gar_bf16_lo(a); v[1] = gar_bf16_hi(a); v[2] = gar_bf16_lo(b); v[3] = gar_bf16_hi(b);
+  v[4] = gar_bf16_lo(c); v[5] = gar_bf16_hi(c); v[6] = gar_bf16_lo(d); v[7] = gar_bf16_hi(d);
+}
+template <> __device__ __forceinline__ void gar_store<1>(gar_io *p, const gar_acc *v) {
+  gar_u16 h;
+  asm("cvt.rn.bf16.f32 %0, %1;" : "=h"(h) : "f"(v[0]));
+  asm volatile("st.global.cs.u16 [%0], %1;" :: "l"(p), "h"(h) : "memory");
+}
+template <> __device__ __forceinline__ void gar_store<2>(gar_io *p, const gar_acc *v) {
+  asm volatile("st.global.cs.u32 [%0], %1;" :: "l"(p), "r"(gar_pack_bf16(v[0], v[1])) : "memory");
+}
+template <> __device__ __forceinline__ void gar_store<4>(gar_io *p, const gar_acc *v) {
+  asm volatile("st.global.cs.v2.u32 [%0], {%1,%2};" :: "l"(p),
+               "r"(gar_pack_bf16(v[0], v[1])), "r"(gar_pack_bf16(v[2], v[3])) : "memory");
+}
+template <> __device__ __forceinline__ void gar_store<8>(gar_io *p, const gar_acc *v) {
+  asm volatile("st.global.cs.v4.u32 [%0], {%1,%2,%3,%4};" :: "l"(p),
+               "r"(gar_pack_bf16(v[0], v[1])), "r"(gar_pack_bf16(v[2], v[3])),
+               "r"(gar_pack_bf16(v[4], v[5])), "r"(gar_pack_bf16(v[6], v[7])) : "memory");
+}
+#else
+template <> __device__ __forceinline__ void gar_load<1>(const gar_io *p, gar_acc *v) {
+  gar_u32 a;
+  asm("ld.global.cs.b32 %0, [%1];" : "=r"(a) : "l"(p));
+  v[0] = *reinterpret_cast<gar_acc *>(&a);
+}
+template <> __device__ __forceinline__ void gar_load<2>(const gar_io *p, gar_acc *v) {
+  gar_u32 a, b;
+  asm("ld.global.cs.v2.b32 {%0,%1}, [%2];" : "=r"(a), "=r"(b) : "l"(p));
+  v[0] = *reinterpret_cast<gar_acc *>(&a); v[1] = *reinterpret_cast<gar_acc *>(&b);
+}
+template <> __device__ __forceinline__ void gar_load<4>(const gar_io *p, gar_acc *v) {
+  gar_u32 a, b, c, d;
+  asm("ld.global.cs.v4.b32 {%0,%1,%2,%3}, [%4];" : "=r"(a), "=r"(b), "=r"(c), "=r"(d) : "l"(p));
+  v[0] = *reinterpret_cast<gar_acc *>(&a); v[1] = *reinterpret_cast<gar_acc *>(&b);
+  v[2] = *reinterpret_cast<gar_acc *>(&c); v[3] = *reinterpret_cast<gar_acc *>(&d);
+}
+template <> __device__ __forceinline__ void gar_store<1>(gar_io *p, const gar_acc *v) {
+  asm volatile("st.global.cs.b32 [%0], %1;" :: "l"(p), "r"(*reinterpret_cast<const gar_u32 *>(&v[0])) : "memory");
+}
+template <> __device__ __forceinline__ void gar_store<2>(gar_io *p, const gar_acc *v) {
+  asm volatile("st.global.cs.v2.b32 [%0], {%1,%2};" :: "l"(p),
+               "r"(*reinterpret_cast<const gar_u32 *>(&v[0])),
+               "r"(*reinterpret_cast<const gar_u32 *>(&v[1])) : "memory");
+}
+template <> __device__ __forceinline__ void gar_store<4>(gar_io *p, const gar_acc *v) {
+  asm volatile("st.global.cs.v4.b32 [%0], {%1,%2,%3,%4};" :: "l"(p),
+               "r"(*reinterpret_cast<const gar_u32 *>(&v[0])),
+               "r"(*reinterpret_cast<const gar_u32 *>(&v[1])),
+               "r"(*reinterpret_cast<const gar_u32 *>(&v[2])),
+               "r"(*reinterpret_cast<const gar_u32 *>(&v[3])) : "memory");
+}
+#endif
+)CUDA";
+
+std::string fmt(const char *f, ...) {
+  char buf[1024];
+  va_list ap;
+  va_start(ap, f);
+  vsnprintf(buf, sizeof buf, f, ap);
+  va_end(ap);
+  return std::string(buf);
+}
+
+// Emission order of one plan's program: results one after another, each by a
+// depth-first walk that evaluates the operand needing more registers first
+// (Sethi-Ullman order), contributions loaded at first use, every result's stores
+// right after it is complete.
+struct Schedule {
+  // items: kind 0 = load leaf j, 1 = combine value v, 2 = store result s
+  std::vector<std::pair<int, int>> items;
+  int peak_live = 0;
+};
+
+Schedule order_program(const FusedProgram &fp) {
+  const int P = fp.P;
+  const int nv = P + (int)fp.a.size();
+  std::vector<int> need(nv, 1);
+  for (int k = 0; k < (int)fp.a.size(); ++k) {
+    const int la = need[fp.a[k]], lb = need[fp.b[k]];
+    need[P + k] = la == lb ? la + 1 : std::max(la, lb);
+  }
+  Schedule sc;
+  std::vector<char> done(nv, 0);
+  std::function<void(int)> visit = [&](int v) {
+    if (done[v]) return;
+    if (v < P) {
+      sc.items.push_back({0, v});
+      done[v] = 1;
+      return;
+    }
+    const int a = fp.a[v - P], b = fp.b[v - P];
+    if (need[b] > need[a]) {
+      visit(b);
+      visit(a);
+    } else {
+      visit(a);
+      visit(b);
+    }
+    sc.items.push_back({1, v});
+    done[v] = 1;
+  };
+  for (int s = 0; s < fp.K; ++s) {
+    visit(fp.out[s]);
+    sc.items.push_back({2, s});
+  }
+  // liveness over this order
+  std::vector<int> last_use(nv, -1), def(nv, -1);
+  for (int t = 0; t < (int)sc.items.size(); ++t) {
+    auto [kind, v] = sc.items[t];
+    if (kind == 0) def[v] = t;
+    if (kind == 1) {
+      def[v] = t;
+      last_use[fp.a[v - P]] = t;
+      last_use[fp.b[v - P]] = t;
+    }
+    if (kind == 2) last_use[fp.out[v]] = t;
+  }
+  std::vector<int> delta(sc.items.size() + 1, 0);
+  for (int v = 0; v < nv; ++v) {
+    if (def[v] < 0) continue;
+    delta[def[v]] += 1;
+    delta[std::max(last_use[v], def[v]) + 1] -= 1;
+  }
+  int live = 0;
+  for (int d : delta) {
+    live += d;
+    sc.peak_live = std::max(sc.peak_live, live);
+  }
+  return sc;
+}
+
+// Largest vector width (elements per thread) that keeps W * peak_live registers of
+// partial results within budget and the load within 16 bytes.
+int choose_width(int dtype, int peak_live, int cap) {
+  const int wmax = std::min(cap, 16 / elem_size(dtype));
+  int w = wmax;
+  while (w > 1 && w * peak_live > 96) w /= 2;
+  return w;
+}
+
+// Emits `template <int W> gar_eval_<tag>(<params>, u64 e0, int b)`: evaluates the program
+// for W consecutive element positions starting at e0, all in block b.  Contribution j is
+// read from row ld_row((b + j) mod P) and result placement p is written to row
+// st_row((b + p) mod P); with rotate == false the rows are j and p themselves (b = 0).
+std::string emit_eval(const FusedProgram &fp, const Schedule &sc, const std::string &tag,
+                      const std::string &params,
+                      const std::function<std::string(const std::string &)> &ld_row,
+                      const std::function<std::string(const std::string &)> &st_row,
+                      bool rotate) {
+  const int P = fp.P;
+  std::string s;
+  s += "template <int W>\nstatic __device__ __forceinline__ void gar_eval_" + tag + "(" + params +
+       ", gar_u64 e0, int b) {\n";
+  s += "  (void)b;\n";
+  auto rank_of = [&](int j) -> std::string {
+    if (!rotate) return std::to_string(j);
+    if (j == 0) return "b";
+    return fmt("(b + %d >= %d ? b + %d : b + %d)", j, P, j - P, j);
+  };
+  // stores of result s go to every placement p whose origin is s
+  std::vector<std::vector<int>> places(fp.K);
+  for (int p = 0; p < P; ++p) places[fp.origin[p]].push_back(p);
+  for (auto [kind, v] : sc.items) {
+    if (kind == 0) {
+      s += fmt("  gar_acc v%d[W]; gar_load<W>(", v) + ld_row(rank_of(v)) + " + e0, v" +
+           std::to_string(v) + ");\n";
+    } else if (kind == 1) {
+      const int a = fp.a[v - P], b = fp.b[v - P];
+      s += fmt("  gar_acc v%d[W];\n#pragma unroll\n  for (int w = 0; w < W; ++w) v%d[w] = gar_op(v%d[w], v%d[w]);\n",
+               v, v, a, b);
+    } else {
+      const int val = fp.out[v];
+      for (int p : places[v])
+        s += "  gar_store<W>(" + st_row(rank_of(p)) + " + e0, v" + std::to_string(val) + ");\n";
+    }
+  }
+  s += "}\n";
+  return s;
+}
+
+std::string dtype_tag(int dtype) { return dtype == GAR_BF16 ? "bf16" : dtype == GAR_I32 ? "i32" : "f32"; }
+std::string op_tag(int op) { return op == GAR_MAX ? "max" : op == GAR_MIN ? "min" : "sum"; }
+
+// Block index of element e for a P-way split of n elements (first n mod P blocks one
+// longer), with all constants compiled in.
+std::string emit_block_of(const std::string &name, int P, uint64_t n) {
+  const uint64_t q = n / P, rem = n % P;
+  std::string s = "static __device__ __forceinline__ int " + name + "(gar_u64 e) {\n";
+  if (q == 0) {
+    s += "  return (int)e;\n";
+  } else {
+    s += fmt("  const gar_u64 big = %lluULL;\n", (unsigned long long)(rem * (q + 1)));
+    s += fmt("  return e < big ? (int)(e / %lluULL) : (int)(%lluULL + (e - big) / %lluULL);\n",
+             (unsigned long long)(q + 1), (unsigned long long)rem, (unsigned long long)q);
+  }
+  s += "}\n";
+  return s;
+}
+
+}  // namespace
+
+CodegenResult generate_fused_source(const gar_plan &pl) {
+  const FusedProgram &fp = pl.prog;
+  const int P = pl.P;
+  Schedule sc = order_program(fp);
+  const int W = choose_width(pl.dtype, sc.peak_live, 16);
+  const bool rotate = pl.K != P;   // latency-optimal results do not depend on the block
+  CodegenResult cg;
+  cg.width = W;
+  cg.kernel_name = fmt("gar_fused_P%d_S%d_K%d_", P, pl.S, pl.K) + dtype_tag(pl.dtype) + "_" +
+                   op_tag(pl.op) + fmt("_W%d", W);
+  std::string s;
+  s += fmt("#define GAR_DTYPE %d\n#define GAR_OP %d\n", pl.dtype, pl.op);
+  s += kSkeleton;
+  s += fmt("#define GAR_P %d\n#define GAR_W %d\n", P, W);
+  s += fmt("#define GAR_N %lluULL\n", (unsigned long long)pl.n);
+  s += fmt("struct gar_args { gar_io *rank[%d]; };\n", P);
+  s += emit_block_of("gar_block_of", P, pl.n);
+  auto row = [](const std::string &r) { return "a.rank[" + r + "]"; };
+  s += emit_eval(fp, sc, "plan", "const gar_args &a", row, row, rotate);
+  s += "extern \"C\" __global__ void __launch_bounds__(256) " + cg.kernel_name +
+       "(const __grid_constant__ gar_args a) {\n";
+  s += "  const gar_u64 nvec = GAR_N / GAR_W;\n";
+  s += "  const gar_u64 stride = (gar_u64)gridDim.x * blockDim.x;\n";
+  s += "  const gar_u64 tid = (gar_u64)blockIdx.x * blockDim.x + threadIdx.x;\n";
+  s += "  for (gar_u64 v = tid; v < nvec; v += stride) {\n";
+  s += "    const gar_u64 e0 = v * GAR_W;\n";
+  if (rotate) {
+    s += "    const int b0 = gar_block_of(e0);\n";
+    s += "    if (GAR_W == 1 || b0 == gar_block_of(e0 + GAR_W - 1)) {\n";
+    s += "      gar_eval_plan<GAR_W>(a, e0, b0);\n";
+    s += "    } else {\n";
+    s += "      for (int w = 0; w < GAR_W; ++w) gar_eval_plan<1>(a, e0 + w, gar_block_of(e0 + w));\n";
+    s += "    }\n";
+  } else {
+    s += "    gar_eval_plan<GAR_W>(a, e0, 0);\n";
+  }
+  s += "  }\n";
+  s += "  const gar_u64 tail = GAR_N - nvec * GAR_W;\n";
+  s += "  if (tid < tail) {\n";
+  s += "    const gar_u64 e = nvec * GAR_W + tid;\n";
+  s += rotate ? "    gar_eval_plan<1>(a, e, gar_block_of(e));\n" : "    gar_eval_plan<1>(a, e, 0);\n";
+  s += "  }\n}\n";
+  cg.source = s;
+  return cg;
+}
+
+CodegenResult generate_batched_source(const std::vector<const gar_plan *> &plans) {
+  const gar_plan &p0 = *plans[0];
+  int peak = 1;
+  std::vector<Schedule> scs;
+  for (const gar_plan *pl : plans) {
+    scs.push_back(order_program(pl->prog));
+    peak = std::max(peak, scs.back().peak_live);
+  }
+  // a row of n elements must split into whole vectors for every row to stay aligned
+  int W = choose_width(p0.dtype, peak, 16);
+  while (W > 1 && p0.n % W != 0) W /= 2;
+  CodegenResult cg;
+  cg.width = W;
+  std::string name = "gar_batched_";
+  for (const gar_plan *pl : plans) name += fmt("P%dS%d_", pl->P, pl->S);
+  cg.kernel_name = name + dtype_tag(p0.dtype) + "_" + op_tag(p0.op) + fmt("_W%d", W);
+  std::string s;
+  s += fmt("#define GAR_DTYPE %d\n#define GAR_OP %d\n", p0.dtype, p0.op);
+  s += kSkeleton;
+  s += fmt("#define GAR_W %d\n#define GAR_N %lluULL\n", W, (unsigned long long)p0.n);
+  s += "struct gar_desc { int plan; int reserved; const void *in; void *out; };\n";
+  s += "struct gar_bargs { const gar_desc *desc; gar_u64 count; };\n";
+  // rows: input row r = in + r * n, output row r = out + r * n.  The generated eval
+  // loads through RIN and stores through ROUT.
+  for (size_t k = 0; k < plans.size(); ++k) {
+    const gar_plan &pl = *plans[k];
+    const bool rotate = pl.K != pl.P;
+    std::string tag = fmt("p%zu", k);
+    s += emit_block_of("gar_block_of_" + tag, pl.P, pl.n);
+    auto ld = [](const std::string &r) { return "(in + GAR_N * (gar_u64)(" + r + "))"; };
+    auto st = [](const std::string &r) { return "(out + GAR_N * (gar_u64)(" + r + "))"; };
+    s += emit_eval(pl.prog, scs[k], tag, "const gar_io *in, gar_io *out", ld, st, rotate);
+  }
+  s += "extern \"C\" __global__ void __launch_bounds__(256) " + cg.kernel_name +
+       "(const __grid_constant__ gar_bargs a) {\n";
+  s += "  const gar_u64 nvec = GAR_N / GAR_W;\n";
+  s += "  const gar_u64 per = nvec + (GAR_N - nvec * GAR_W);\n";
+  s += "  const gar_u64 total = a.count * per;\n";
+  s += "  const gar_u64 stride = (gar_u64)gridDim.x * blockDim.x;\n";
+  s += "  for (gar_u64 g = (gar_u64)blockIdx.x * blockDim.x + threadIdx.x; g < total; g += stride) {\n";
+  s += "    const gar_u64 i = g / per, v = g - i * per;\n";
+  s += "    const gar_desc d = a.desc[i];\n";
+  s += "    const gar_io *in = (const gar_io *)d.in;\n";
+  s += "    gar_io *out = (gar_io *)d.out;\n";
+  s += "    const bool aligned = (((gar_u64)in | (gar_u64)out) & (GAR_W * sizeof(gar_io) - 1)) == 0;\n";
+  s += "    switch (d.plan) {\n";
+  for (size_t k = 0; k < plans.size(); ++k) {
+    const gar_plan &pl = *plans[k];
+    const bool rotate = pl.K != pl.P;
+    std::string tag = fmt("p%zu", k);
+    std::string bo = "gar_block_of_" + tag;
+    s += fmt("    case %zu:\n", k);
+    s += "      if (v < nvec) {\n";
+    s += "        const gar_u64 e0 = v * GAR_W;\n";
+    if (rotate) {
+      s += "        const int b0 = " + bo + "(e0);\n";
+      s += "        if (aligned && (GAR_W == 1 || b0 == " + bo + "(e0 + GAR_W - 1))) gar_eval_" + tag +
+           "<GAR_W>(in, out, e0, b0);\n";
+      s += "        else for (int w = 0; w < GAR_W; ++w) gar_eval_" + tag + "<1>(in, out, e0 + w, " + bo +
+           "(e0 + w));\n";
+    } else {
+      s += "        if (aligned) gar_eval_" + tag + "<GAR_W>(in, out, e0, 0);\n";
+      s += "        else for (int w = 0; w < GAR_W; ++w) gar_eval_" + tag + "<1>(in, out, e0 + w, 0);\n";
+    }
+    s += "      } else {\n";
+    s += "        const gar_u64 e = nvec * GAR_W + (v - nvec);\n";
+    s += rotate ? "        gar_eval_" + tag + "<1>(in, out, e, " + bo + "(e));\n"
+                : "        gar_eval_" + tag + "<1>(in, out, e, 0);\n";
+    s += "      }\n      break;\n";
+  }
+  s += "    default: break;\n    }\n  }\n}\n";
+  cg.source = s;
+  return cg;
+}
+
+}  // namespace gar

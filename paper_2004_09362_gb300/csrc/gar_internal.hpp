@@ -1,0 +1,135 @@
+// Internal definitions shared by the schedule builder, the code generator, the
+// kernels and the C ABI.  Not part of the public interface (include/gar.h).
+#pragma once
+
+#include <cstdint>
+#include <cstddef>
+#include <string>
+#include <vector>
+
+#include "../../include/gar.h"
+
+namespace gar {
+
+// Buffers a step-faithful op reads or writes, per rank.
+enum Buf : uint8_t {
+  BUF_NONE = 0,
+  BUF_RANK = 1,  // the caller's rank buffer (input, then output), element type T
+  BUF_QP0 = 2,   // q' slots, ping (accumulation type)
+  BUF_QP1 = 3,   // q' slots, pong
+  BUF_QS = 4     // q* slots (accumulation type)
+};
+constexpr int NUM_WS_BUFS = 3;  // QP0, QP1, QS
+
+// One block operation of a step-faithful launch, identical for every rank x.  With
+// b = (x - dst_place) mod P (the block index, which a move never changes):
+//   recv  = buf[recv_buf][(x + partner) mod P][block b]          (if recv_place >= 0)
+//   out_k = own(buf[out_k_own][x][block b]) (+) recv  ->  buf[out_k_buf][x][block b]
+// A missing own operand makes out_k a copy of recv; a missing recv a copy of own.
+struct StepOp {
+  int16_t recv_place;  // placement of the received vector at the partner, -1 = none
+  int16_t dst_place;   // placement at this rank
+  uint8_t recv_buf;
+  uint8_t out0_buf, out0_own;
+  uint8_t out1_buf, out1_own;
+  uint8_t pad[7];
+};
+static_assert(sizeof(StepOp) == 16, "StepOp must stay 16 bytes");
+
+struct Launch {
+  int phase;         // 0 reduction step, 1 distribution step, 2 local finalize copy
+  int comm_step;     // index of the communication step it implements, -1 for local
+  int partner;       // rank x receives from (x + partner) mod P
+  int first_op;      // into Plan::ops
+  int nops;
+};
+
+struct CommStep {
+  int phase;                      // 0 reduce, 1 distribute
+  int i;                          // the paper's step index i
+  int N, d;
+  int partner;
+  std::vector<int32_t> tx;        // placements transmitted by every rank
+  uint64_t msg_bytes;             // predicted, all ranks together
+};
+
+// Per-element-position program of the fused mode.
+struct FusedProgram {
+  int P = 0, K = 0;
+  std::vector<int32_t> a, b;      // combine k: value P + k = a[k] (+) b[k]
+  std::vector<int32_t> out;       // out[s] = value id of result copy s
+  std::vector<int32_t> origin;    // origin[p] = copy written to placement p
+};
+
+struct JitKernel;  // jit.cpp
+
+}  // namespace gar
+
+struct gar_plan {
+  int P = 0, L = 0, S = 0, r = 0, K = 0;
+  uint64_t n = 0;
+  int dtype = 0, op = 0;
+  uint64_t q = 0, rem = 0;        // block i has q + (i < rem) elements
+  std::vector<int> N;             // N_0..N_L
+  std::vector<gar::CommStep> comm;
+  std::vector<gar::StepOp> ops;
+  std::vector<gar::Launch> launches;
+  bool ws_used[gar::NUM_WS_BUFS] = {false, false, false};
+  uint64_t n_pad = 0;             // per-rank stride of workspace slices (elements)
+  size_t ws_bytes = 0;
+  gar::FusedProgram prog;
+
+  // device state
+  void *ws = nullptr;
+  size_t ws_set_bytes = 0;
+  int device = -1;
+  gar::StepOp *d_ops = nullptr;
+  unsigned long long *d_step_bytes = nullptr;
+  gar_stream_t last_stream = nullptr;
+  bool ran_step_faithful = false;
+  gar::JitKernel *fused = nullptr;   // owned by the JIT cache
+  int fused_width = 0;
+};
+
+namespace gar {
+
+int elem_size(int dtype);
+int acc_size(int dtype);
+int ceil_log2(int P);
+
+// plan.cpp
+int build_plan(gar_plan *pl);
+
+// codegen.cpp
+struct CodegenResult {
+  std::string source;
+  std::string kernel_name;
+  int width = 1;
+};
+CodegenResult generate_fused_source(const gar_plan &pl);
+CodegenResult generate_batched_source(const std::vector<const gar_plan *> &plans);
+
+// jit.cpp
+struct JitKernel {
+  void *library = nullptr;   // cudaLibrary_t
+  void *kernel = nullptr;    // cudaKernel_t
+  std::vector<char> cubin;
+  std::string name;
+  int width = 1;
+  int threads = 256;
+  int blocks_per_sm = 0;
+  bool loaded = false;
+};
+int jit_compile(const CodegenResult &cg, JitKernel **out);
+int jit_load(JitKernel *k);
+
+// step_kernels.cu
+int launch_step(const gar_plan &pl, const Launch &ln, int launch_index, void *const *rank,
+                gar_stream_t stream);
+
+// api.cpp
+void set_error(const std::string &msg);
+const char *last_error_cstr();
+int cuda_fail(int err, const char *what);
+
+}  // namespace gar

@@ -1,0 +1,272 @@
+// Step-faithful mode: one kernel launch per communication step of the schedule.
+//
+// A launch applies the step's block ops (plan.cpp) for every rank x at once.  An op
+// names a placement; rank x works on block b = (x - dst_place) mod P, which is the same
+// block index at the partner (a move by t^{l} changes a vector's placement, never its
+// block index; eq. comm_op_0).  "Sending" is a coalesced 16-byte vector read of the
+// partner rank's block; the read value is combined in registers with the own block
+// (eq. distr_vectors_combination) and stored.  Every CTA owns one chunk of one block
+// of one (op, rank) pair.  Each warp counts the elements it read from partners and adds
+// the bytes to the step's counter, so the bytes a step actually moved are recorded.
+#include <cuda_bf16.h>
+#include <cuda_runtime.h>
+
+#include <cstdint>
+
+#include "gar_internal.hpp"
+
+namespace gar {
+namespace {
+
+constexpr int kThreads = 256;
+constexpr uint64_t kChunk = 8192;  // elements per CTA
+
+template <int MAXP>
+struct StepArgs {
+  void *rank[MAXP];
+  void *ws[NUM_WS_BUFS];             // QP0, QP1, QS slice bases (nullptr if unused)
+  const StepOp *ops;                 // this launch's ops
+  unsigned long long *bytes;         // counter of the communication step, or nullptr
+  uint64_t q, rem, n_pad;
+  int P, partner, nops, nchunks;
+};
+
+template <typename T> struct AccOf { using type = T; };
+template <> struct AccOf<__nv_bfloat16> { using type = float; };
+
+__device__ __forceinline__ float widen(__nv_bfloat16 x) { return __bfloat162float(x); }
+__device__ __forceinline__ float widen(float x) { return x; }
+__device__ __forceinline__ int widen(int x) { return x; }
+__device__ __forceinline__ void narrow(float x, __nv_bfloat16 *o) { *o = __float2bfloat16_rn(x); }
+__device__ __forceinline__ void narrow(float x, float *o) { *o = x; }
+__device__ __forceinline__ void narrow(int x, int *o) { *o = x; }
+
+template <int OP> __device__ __forceinline__ float combine(float a, float b) {
+  if (OP == GAR_SUM) return a + b;
+  if (OP == GAR_MAX) return fmaxf(a, b);
+  return fminf(a, b);
+}
+template <int OP> __device__ __forceinline__ int combine(int a, int b) {
+  if (OP == GAR_SUM) return (int)((unsigned)a + (unsigned)b);
+  if (OP == GAR_MAX) return a > b ? a : b;
+  return a < b ? a : b;
+}
+
+// One element / four aligned elements of buffer `buf` (rank buffers hold T, workspace
+// slices hold the accumulation type A).
+template <typename T, typename A>
+__device__ __forceinline__ A load1(uint8_t buf, const void *base, uint64_t e) {
+  if (buf == BUF_RANK) return widen(static_cast<const T *>(base)[e]);
+  return static_cast<const A *>(base)[e];
+}
+
+template <typename T, typename A>
+__device__ __forceinline__ void load4(uint8_t buf, const void *base, uint64_t e, A (&v)[4]) {
+  if (buf == BUF_RANK && sizeof(T) == 2) {
+    const uint2 u = *reinterpret_cast<const uint2 *>(static_cast<const T *>(base) + e);
+    v[0] = (A)__uint_as_float(u.x << 16);
+    v[1] = (A)__uint_as_float(u.x & 0xffff0000u);
+    v[2] = (A)__uint_as_float(u.y << 16);
+    v[3] = (A)__uint_as_float(u.y & 0xffff0000u);
+  } else {
+    const A *p = (buf == BUF_RANK) ? reinterpret_cast<const A *>(static_cast<const T *>(base))
+                                   : static_cast<const A *>(base);
+    const int4 u = *reinterpret_cast<const int4 *>(p + e);
+    v[0] = *reinterpret_cast<const A *>(&u.x);
+    v[1] = *reinterpret_cast<const A *>(&u.y);
+    v[2] = *reinterpret_cast<const A *>(&u.z);
+    v[3] = *reinterpret_cast<const A *>(&u.w);
+  }
+}
+
+template <typename T, typename A>
+__device__ __forceinline__ void store1(uint8_t buf, void *base, uint64_t e, A v) {
+  if (buf == BUF_RANK)
+    narrow(v, static_cast<T *>(base) + e);
+  else
+    static_cast<A *>(base)[e] = v;
+}
+
+template <typename T, typename A>
+__device__ __forceinline__ void store4(uint8_t buf, void *base, uint64_t e, const A (&v)[4]) {
+  if (buf == BUF_RANK && sizeof(T) == 2) {
+    __nv_bfloat16 h[4];
+#pragma unroll
+    for (int k = 0; k < 4; ++k) narrow(v[k], &h[k]);
+    uint2 u;
+    u.x = (uint32_t)__bfloat16_as_ushort(h[0]) | ((uint32_t)__bfloat16_as_ushort(h[1]) << 16);
+    u.y = (uint32_t)__bfloat16_as_ushort(h[2]) | ((uint32_t)__bfloat16_as_ushort(h[3]) << 16);
+    *reinterpret_cast<uint2 *>(static_cast<T *>(base) + e) = u;
+  } else {
+    A *p = (buf == BUF_RANK) ? reinterpret_cast<A *>(static_cast<T *>(base)) : static_cast<A *>(base);
+    int4 u;
+    u.x = *reinterpret_cast<const int *>(&v[0]);
+    u.y = *reinterpret_cast<const int *>(&v[1]);
+    u.z = *reinterpret_cast<const int *>(&v[2]);
+    u.w = *reinterpret_cast<const int *>(&v[3]);
+    *reinterpret_cast<int4 *>(p + e) = u;
+  }
+}
+
+template <typename A, int MAXP>
+__device__ __forceinline__ void *buf_ptr(const StepArgs<MAXP> &a, uint8_t buf, int rank) {
+  if (buf == BUF_RANK) return a.rank[rank];
+  if (buf == BUF_NONE) return nullptr;
+  return static_cast<char *>(a.ws[buf - BUF_QP0]) + (uint64_t)rank * a.n_pad * sizeof(A);
+}
+
+template <typename T, int OP, int MAXP>
+__global__ void __launch_bounds__(kThreads) step_kernel(const __grid_constant__ StepArgs<MAXP> a) {
+  using A = typename AccOf<T>::type;
+  uint64_t bid = blockIdx.x;
+  const int chunk = (int)(bid % (uint64_t)a.nchunks);
+  bid /= (uint64_t)a.nchunks;
+  const int x = (int)(bid % (uint64_t)a.P);
+  const int oi = (int)(bid / (uint64_t)a.P);
+  if (oi >= a.nops) return;
+  const StepOp op = a.ops[oi];
+  const int b = ((x - (int)op.dst_place) % a.P + a.P) % a.P;
+  const uint64_t bstart = (uint64_t)b * a.q + ((uint64_t)b < a.rem ? (uint64_t)b : a.rem);
+  const uint64_t blen = a.q + ((uint64_t)b < a.rem ? 1 : 0);
+  const uint64_t c0 = (uint64_t)chunk * kChunk;
+  if (c0 >= blen) return;
+  const uint64_t lo = bstart + c0;
+  const uint64_t hi = bstart + (blen < c0 + kChunk ? blen : c0 + kChunk);
+
+  const bool has_recv = op.recv_place >= 0;
+  const int partner = ((x + a.partner) % a.P + a.P) % a.P;
+  const void *recv = has_recv ? buf_ptr<A>(a, op.recv_buf, partner) : nullptr;
+  void *out0 = buf_ptr<A>(a, op.out0_buf, x);
+  const void *own0 = buf_ptr<A>(a, op.out0_own, x);
+  void *out1 = buf_ptr<A>(a, op.out1_buf, x);
+  const void *own1 = buf_ptr<A>(a, op.out1_own, x);
+
+  uint64_t moved = 0;
+  auto do1 = [&](uint64_t e) {
+    A r = A(0);
+    if (has_recv) {
+      r = load1<T, A>(op.recv_buf, recv, e);
+      ++moved;
+    }
+    A o0 = r, o1 = r;
+    if (own0) o0 = has_recv ? combine<OP>(load1<T, A>(op.out0_own, own0, e), r) : load1<T, A>(op.out0_own, own0, e);
+    if (out1 && own1) o1 = has_recv ? combine<OP>(load1<T, A>(op.out1_own, own1, e), r) : load1<T, A>(op.out1_own, own1, e);
+    store1<T, A>(op.out0_buf, out0, e, o0);
+    if (out1) store1<T, A>(op.out1_buf, out1, e, o1);
+  };
+  auto do4 = [&](uint64_t e) {
+    A r[4] = {A(0), A(0), A(0), A(0)};
+    if (has_recv) {
+      load4<T, A>(op.recv_buf, recv, e, r);
+      moved += 4;
+    }
+    A o0[4], o1[4];
+    if (own0) {
+      load4<T, A>(op.out0_own, own0, e, o0);
+      if (has_recv)
+#pragma unroll
+        for (int k = 0; k < 4; ++k) o0[k] = combine<OP>(o0[k], r[k]);
+    } else {
+#pragma unroll
+      for (int k = 0; k < 4; ++k) o0[k] = r[k];
+    }
+    if (out1) {
+      if (own1) {
+        load4<T, A>(op.out1_own, own1, e, o1);
+        if (has_recv)
+#pragma unroll
+          for (int k = 0; k < 4; ++k) o1[k] = combine<OP>(o1[k], r[k]);
+      } else {
+#pragma unroll
+        for (int k = 0; k < 4; ++k) o1[k] = r[k];
+      }
+    }
+    store4<T, A>(op.out0_buf, out0, e, o0);
+    if (out1) store4<T, A>(op.out1_buf, out1, e, o1);
+  };
+
+  // Element offsets are the same in every buffer, and every buffer base is 16-byte
+  // aligned, so one head/body/tail split serves all operands.
+  uint64_t va = (lo + 3) & ~uint64_t(3);
+  uint64_t vb = hi & ~uint64_t(3);
+  if (va > hi) va = hi;
+  if (vb < va) vb = va;
+  for (uint64_t e = lo + threadIdx.x; e < va; e += blockDim.x) do1(e);
+  for (uint64_t e = va + 4 * (uint64_t)threadIdx.x; e < vb; e += 4 * (uint64_t)blockDim.x) do4(e);
+  for (uint64_t e = vb + threadIdx.x; e < hi; e += blockDim.x) do1(e);
+
+  if (a.bytes != nullptr && has_recv) {
+    unsigned long long m = moved;
+#pragma unroll
+    for (int off = 16; off > 0; off >>= 1) m += __shfl_down_sync(0xffffffffu, m, off);
+    const unsigned long long esize = (op.recv_buf == BUF_RANK) ? sizeof(T) : sizeof(A);
+    if ((threadIdx.x & 31) == 0 && m) atomicAdd(a.bytes, m * esize);
+  }
+}
+
+template <typename T, int OP, int MAXP>
+int launch_typed(const gar_plan &pl, const Launch &ln, int launch_index, void *const *rank,
+                 gar_stream_t stream) {
+  (void)launch_index;
+  StepArgs<MAXP> a{};
+  for (int x = 0; x < pl.P; ++x) a.rank[x] = rank[x];
+  int slot = 0;
+  for (int k = 0; k < NUM_WS_BUFS; ++k) {
+    if (pl.ws_used[k]) {
+      a.ws[k] = static_cast<char *>(pl.ws) + (size_t)slot * pl.P * pl.n_pad * acc_size(pl.dtype);
+      ++slot;
+    } else {
+      a.ws[k] = nullptr;
+    }
+  }
+  a.ops = pl.d_ops + ln.first_op;
+  a.bytes = (ln.comm_step >= 0) ? pl.d_step_bytes + ln.comm_step : nullptr;
+  a.q = pl.q;
+  a.rem = pl.rem;
+  a.n_pad = pl.n_pad;
+  a.P = pl.P;
+  a.partner = ln.partner;
+  a.nops = ln.nops;
+  const uint64_t maxblk = pl.q + (pl.rem ? 1 : 0);
+  a.nchunks = (int)((maxblk + kChunk - 1) / kChunk);
+  if (a.nchunks == 0 || ln.nops == 0) return GAR_OK;
+  const uint64_t grid = (uint64_t)a.nchunks * (uint64_t)pl.P * (uint64_t)ln.nops;
+  if (grid > 0x7fffffffull) {
+    set_error("step launch grid too large");
+    return GAR_EINVAL;
+  }
+  step_kernel<T, OP, MAXP><<<(unsigned)grid, kThreads, 0, (cudaStream_t)stream>>>(a);
+  cudaError_t e = cudaGetLastError();
+  if (e != cudaSuccess) return cuda_fail(e, "step kernel launch");
+  return GAR_OK;
+}
+
+template <typename T, int MAXP>
+int launch_op(const gar_plan &pl, const Launch &ln, int li, void *const *rank, gar_stream_t s) {
+  switch (pl.op) {
+    case GAR_SUM: return launch_typed<T, GAR_SUM, MAXP>(pl, ln, li, rank, s);
+    case GAR_MAX: return launch_typed<T, GAR_MAX, MAXP>(pl, ln, li, rank, s);
+    case GAR_MIN: return launch_typed<T, GAR_MIN, MAXP>(pl, ln, li, rank, s);
+  }
+  return GAR_EINVAL;
+}
+
+template <int MAXP>
+int launch_dt(const gar_plan &pl, const Launch &ln, int li, void *const *rank, gar_stream_t s) {
+  switch (pl.dtype) {
+    case GAR_F32: return launch_op<float, MAXP>(pl, ln, li, rank, s);
+    case GAR_BF16: return launch_op<__nv_bfloat16, MAXP>(pl, ln, li, rank, s);
+    case GAR_I32: return launch_op<int, MAXP>(pl, ln, li, rank, s);
+  }
+  return GAR_EINVAL;
+}
+
+}  // namespace
+
+int launch_step(const gar_plan &pl, const Launch &ln, int launch_index, void *const *rank,
+                gar_stream_t stream) {
+  if (pl.P <= 128) return launch_dt<128>(pl, ln, launch_index, rank, stream);
+  return launch_dt<GAR_MAX_P>(pl, ln, launch_index, rank, stream);
+}
+
+}  // namespace gar

@@ -1,0 +1,360 @@
+"""GPU parity: libgar's CUDA kernels (through the C ABI) against the CPU oracle.
+
+Floating-point results follow the schedule's association order, so every comparison
+with the oracle is bit-exact, for fp32, bf16 (fp32 accumulation) and int32, in both
+modes.  Full-size workloads are compared on sampled element positions (the oracle
+runs on an element subset) and, everywhere, against properties that hold at any size:
+max/min equal the column max/min exactly, and sums lie within the tree error bound
+L * 2^-24 * sum|x| of a float64 reference (plus one bf16 rounding, 2^-8 relative).
+"""
+
+import numpy as np
+import pytest
+import torch
+
+import gar_inputs
+from oracle import gar_oracle as G
+
+pytestmark = pytest.mark.gpu
+
+gar = pytest.importorskip("paper_2004_09362_gb300.gar")
+
+DEV = "cuda"
+
+
+def _Ss(P):
+    L = G.ceil_log2(P)
+    return list(range(L, 2 * L + 1))
+
+
+def _np_inputs(P, n, dtype, seed, dist=None):
+    if dist is None:
+        dist = ("int", -1000, 1000) if dtype == "i32" else ("normal", 0.0, 1.0)
+    t = gar_inputs.rank_inputs(P, n, dtype, dist, seed)
+    return t
+
+
+def _to_host_list(t, dtype):
+    if dtype == "bf16":
+        t = t.float()
+    return [t[x].numpy().copy() for x in range(t.shape[0])]
+
+
+def _padded_device(t):
+    """Copy a [P, n] tensor to the GPU with a row stride that keeps every row 16-byte
+    aligned; returns (storage, row view)."""
+    P, n = t.shape
+    per16 = 16 // t.element_size()
+    n_pad = max(per16, (n + per16 - 1) // per16 * per16)
+    store = torch.zeros((P, n_pad), dtype=t.dtype, device=DEV)
+    store[:, :n] = t.to(DEV)
+    return store, store[:, :n]
+
+
+def _run(plan, t, mode):
+    store, view = _padded_device(t)
+    gar.gar_allreduce(plan, store, mode)
+    torch.cuda.synchronize()
+    return view.cpu()
+
+
+def _bits(a):
+    a = np.ascontiguousarray(a)
+    return a.view(np.uint32) if a.dtype.itemsize == 4 else a.view(np.uint16)
+
+
+def _assert_same(got_t, want_list, dtype, what=""):
+    got = _to_host_list(got_t, dtype)
+    for x in range(len(want_list)):
+        g, w = got[x], want_list[x].astype(got[x].dtype)
+        if not np.array_equal(_bits(g), _bits(w)):
+            bad = np.nonzero(_bits(g) != _bits(w))[0]
+            raise AssertionError(f"{what} rank {x}: {len(bad)} mismatches, first at {bad[:5]}: "
+                                 f"got {g[bad[:5]]} want {w[bad[:5]]}")
+
+
+# ---------------------------------------------------------------------------
+# Exhaustive small cases: every P up to 17, every step count, ragged n
+# ---------------------------------------------------------------------------
+
+@pytest.mark.parametrize("P", list(range(1, 18)) + [24, 31, 32, 33])
+@pytest.mark.parametrize("mode", ["fused", "step"])
+def test_small_every_step_count(P, mode):
+    """fp32 at ragged sizes around the block and vector boundaries; int32 and bf16 at
+    one ragged size; every step count."""
+    cases = [(n, "f32") for n in sorted({0, 1, P + 1, 1031})]
+    cases += [(4 * P + 3, dt) for dt in ("f32", "i32", "bf16")]
+    for (n, dtype) in cases:
+        t = _np_inputs(P, n, dtype, seed=P * 1000 + n)
+        host = _to_host_list(t, dtype)
+        for S in _Ss(P):
+            plan = gar.gar_plan_create(P, n, dtype, "sum", S)
+            got = _run(plan, t, mode)
+            want = G.allreduce(host, S, "sum", dtype)
+            _assert_same(got, want, dtype, f"P={P} n={n} {dtype} S={S} {mode}")
+
+
+@pytest.mark.parametrize("op", ["max", "min"])
+@pytest.mark.parametrize("mode", ["fused", "step"])
+def test_small_max_min(op, mode):
+    for P in (2, 3, 5, 6, 7, 8, 12, 13):
+        n = 3 * P + 5
+        for dtype in ("f32", "i32", "bf16"):
+            t = _np_inputs(P, n, dtype, seed=7 * P)
+            host = _to_host_list(t, dtype)
+            ref = G.column_reduce_exact(host, op, dtype)
+            for S in _Ss(P):
+                plan = gar.gar_plan_create(P, n, dtype, op, S)
+                got = _run(plan, t, mode)
+                _assert_same(got, [ref] * P, dtype, f"{op} P={P} {dtype} S={S} {mode}")
+
+
+# ---------------------------------------------------------------------------
+# The paper-shaped workloads at sizes the oracle finishes in seconds
+# ---------------------------------------------------------------------------
+
+@pytest.mark.parametrize("mode", ["fused", "step"])
+def test_p5_f32_and_i32(mode):
+    wl = gar_inputs.WORKLOADS["p5_f32"]
+    t = gar_inputs.rank_inputs(wl.P, wl.n, wl.dtype, wl.dist, wl.seed)
+    host = _to_host_list(t, "f32")
+    for S in wl.steps:
+        plan = gar.gar_plan_create(wl.P, wl.n, "f32", "sum", S)
+        _assert_same(_run(plan, t, mode), G.allreduce(host, S, "sum", "f32"), "f32", f"S={S}")
+    wl = gar_inputs.WORKLOADS["p5_i32"]
+    t = gar_inputs.rank_inputs(wl.P, wl.n, wl.dtype, wl.dist, wl.seed)
+    host = _to_host_list(t, "i32")
+    for op in wl.ops:
+        for S in wl.steps:
+            plan = gar.gar_plan_create(wl.P, wl.n, "i32", op, S)
+            _assert_same(_run(plan, t, mode), G.allreduce(host, S, op, "i32"), "i32", f"{op} S={S}")
+
+
+@pytest.mark.parametrize("mode", ["fused", "step"])
+def test_p8_1mib_every_step_count(mode):
+    wl = gar_inputs.WORKLOADS["p8_1mib_f32"]
+    t = gar_inputs.rank_inputs(wl.P, wl.n, wl.dtype, wl.dist, wl.seed)
+    host = _to_host_list(t, "f32")
+    for S in wl.steps:
+        plan = gar.gar_plan_create(wl.P, wl.n, "f32", "sum", S)
+        _assert_same(_run(plan, t, mode), G.allreduce(host, S, "sum", "f32"), "f32", f"S={S}")
+
+
+@pytest.mark.parametrize("mode", ["fused", "step"])
+def test_p127_bf16_reduced_n(mode):
+    """P=127 bf16 with fp32 accumulation at a ragged n that spans several vector widths
+    per block; every step count 7..14."""
+    P, n = 127, 127 * 40 + 19
+    t = gar_inputs.rank_inputs(P, n, "bf16", ("normal", 0.0, 1.0), 99)
+    host = _to_host_list(t, "bf16")
+    for S in range(7, 15):
+        plan = gar.gar_plan_create(P, n, "bf16", "sum", S)
+        _assert_same(_run(plan, t, mode), G.allreduce(host, S, "sum", "bf16"), "bf16", f"S={S}")
+
+
+# ---------------------------------------------------------------------------
+# Recorded step bytes equal the schedule's predicted volume
+# ---------------------------------------------------------------------------
+
+@pytest.mark.parametrize("P,n,dtype", [(5, 1024, "f32"), (8, 262144, "f32"), (7, 1001, "bf16"),
+                                       (24, 24 * 1000 + 7, "f32"), (127, 5000, "bf16")])
+def test_recorded_step_bytes(P, n, dtype):
+    t = _np_inputs(P, n, dtype, seed=5)
+    for S in _Ss(P):
+        plan = gar.gar_plan_create(P, n, dtype, "sum", S)
+        _run(plan, t, "step")
+        rec = gar.gar_last_step_bytes(plan)
+        _ws, pred, _S = gar.gar_plan_bytes(plan)
+        run = G.simulate(P, n, S, dtype=dtype)
+        assert rec == pred == run.step_bytes(), (P, S, rec, pred)
+
+
+# ---------------------------------------------------------------------------
+# Full sizes, in the launch configuration bench.py times
+# ---------------------------------------------------------------------------
+
+def _sample(n, P, k=4096, seed=0):
+    rng = np.random.default_rng(seed)
+    bounds = G.block_bounds(n, P)
+    picks = [rng.integers(0, n, k)]
+    for (lo, hi) in bounds:                       # both ends of every block
+        if hi > lo:
+            picks.append(np.array([lo, min(lo + 1, hi - 1), max(hi - 2, lo), hi - 1]))
+    picks.append(np.array([0, n - 1]))
+    return np.unique(np.concatenate(picks))
+
+
+def _tree_bound_check(got_rows, inp, L, dtype):
+    """Property at any size: |result - exact| <= L 2^-24 sum|x| (+ 2^-8 |exact| for bf16)."""
+    x64 = inp.to(DEV, torch.float64)
+    exact = x64.sum(0)
+    mag = x64.abs().sum(0)
+    tol = L * 2.0 ** -24 * mag * 1.0001
+    if dtype == "bf16":
+        tol = tol + 2.0 ** -8 * exact.abs()
+    for r in range(got_rows.shape[0]):
+        err = (got_rows[r].to(torch.float64) - exact).abs()
+        assert bool((err <= tol + 1e-30).all()), f"rank {r}: max excess {(err - tol).max().item()}"
+
+
+@pytest.mark.parametrize("mode", ["fused", "step"])
+def test_full_p24_64mib(mode):
+    wl = gar_inputs.WORKLOADS["p24_64mib_f32"]
+    P, n = wl.P, wl.n
+    inp = gar_inputs.rank_inputs(P, n, wl.dtype, wl.dist, wl.seed, device=DEV)
+    buf = inp.clone()
+    plan = gar.gar_plan_create(P, n, "f32", "sum", 10)
+    gar.gar_allreduce(plan, buf, mode)
+    torch.cuda.synchronize()
+    # bandwidth-optimal: every rank holds identical bits
+    assert bool((buf == buf[0:1]).all())
+    _tree_bound_check(buf, inp, 5, "f32")
+    idx = _sample(n, P)
+    host_in = [inp[x, torch.from_numpy(idx).to(DEV)].cpu().numpy() for x in range(P)]
+    # oracle on the sampled element positions: rebuild full-length vectors lazily by
+    # running it on the subset (elementwise => exact)
+    full = [np.zeros(n, np.float32) for _ in range(P)]
+    for x in range(P):
+        full[x][idx] = host_in[x]
+    want = G.allreduce(full, 10, "sum", "f32", elements=idx)
+    got = buf[:, torch.from_numpy(idx).to(DEV)].cpu().numpy()
+    for x in range(P):
+        np.testing.assert_array_equal(got[x].view(np.uint32), want[x].view(np.uint32))
+    if mode == "step":
+        rec = gar.gar_last_step_bytes(plan)
+        _ws, pred, _S = gar.gar_plan_bytes(plan)
+        assert rec == pred
+
+
+@pytest.mark.parametrize("S", [7, 10, 14])
+@pytest.mark.parametrize("mode", ["fused", "step"])
+def test_full_p127_8mib_bf16(S, mode):
+    wl = gar_inputs.WORKLOADS["p127_8mib_bf16"]
+    P, n = wl.P, wl.n
+    inp = gar_inputs.rank_inputs(P, n, wl.dtype, wl.dist, wl.seed, device=DEV)
+    buf = inp.clone()
+    plan = gar.gar_plan_create(P, n, "bf16", "sum", S)
+    gar.gar_allreduce(plan, buf, mode)
+    torch.cuda.synchronize()
+    _tree_bound_check(buf.float(), inp.float(), 7, "bf16")
+    idx = _sample(n, P, k=512, seed=S)
+    sel = torch.from_numpy(idx).to(DEV)
+    sub = inp[:, sel].float().cpu().numpy()
+    full = [np.zeros(n, np.float32) for _ in range(P)]
+    for x in range(P):
+        full[x][idx] = sub[x]
+    want = G.allreduce(full, S, "sum", "bf16", elements=idx)
+    got = buf[:, sel].float().cpu().numpy()
+    for x in range(P):
+        np.testing.assert_array_equal(got[x].view(np.uint32), want[x].view(np.uint32))
+
+
+# ---------------------------------------------------------------------------
+# Batched small Allreduces (65536 instances of P=6 / P=7, 106 fp32 per rank)
+# ---------------------------------------------------------------------------
+
+def _batched_setup(count, Ps, n, seed, op, steps="lo"):
+    flat, layout = gar_inputs.batched_inputs(count, Ps, n, "f32", ("normal", 0.0, 1.0), seed,
+                                             device=DEV)
+    out = torch.empty_like(flat)
+    plans = [gar.gar_plan_create(P, n, "f32", op, gar.GAR_STEPS_LO if steps == "lo" else steps)
+             for P in Ps]
+    idx = {P: k for k, P in enumerate(Ps)}
+    es = flat.element_size()
+    desc = gar.make_batch_desc([idx[P] for (P, _o) in layout],
+                               [flat.data_ptr() + o * es for (_P, o) in layout],
+                               [out.data_ptr() + o * es for (_P, o) in layout])
+    return flat, out, layout, plans, desc
+
+
+@pytest.mark.parametrize("op", ["sum", "max"])
+def test_batched_425_bytes(op):
+    count, Ps, n = 65536, (6, 7), 106
+    flat, out, layout, plans, desc = _batched_setup(count, Ps, n, 1236, op)
+    gar.gar_allreduce_batched(plans, desc, count)
+    torch.cuda.synchronize()
+    rng = np.random.default_rng(1)
+    check = np.unique(np.concatenate([[0, count // 2 - 1, count // 2, count - 1],
+                                      rng.integers(0, count, 200)]))
+    fh, oh = flat.cpu().numpy(), out.cpu().numpy()
+    for i in check:
+        P, off = layout[i]
+        xs = [fh[off + x * n: off + (x + 1) * n].copy() for x in range(P)]
+        want = G.allreduce(xs, G.ceil_log2(P), op, "f32")
+        for x in range(P):
+            got = oh[off + x * n: off + (x + 1) * n]
+            np.testing.assert_array_equal(got.view(np.uint32), want[x].view(np.uint32))
+    # every instance: property check against float64 / exact max
+    for P in Ps:
+        offs = np.array([o for (p, o) in layout if p == P])
+        base = torch.from_numpy(offs).to(DEV)
+        ar = torch.arange(P * n, device=DEV)
+        gi = (base[:, None] + ar[None, :]).view(-1, P, n)
+        xin, xout = flat[gi], out[gi]
+        if op == "max":
+            assert bool((xout == xin.max(1, keepdim=True).values).all())
+        else:
+            x64 = xin.double()
+            tol = 3 * 2.0 ** -24 * x64.abs().sum(1, keepdim=True) * 1.0001
+            assert bool(((xout.double() - x64.sum(1, keepdim=True)).abs() <= tol + 1e-30).all())
+
+
+def test_batched_mixed_order_and_steps():
+    """Instances of different plans interleaved, intermediate step counts, in == out, and
+    a misaligned instance (handled element-wise)."""
+    n = 50
+    Ps = (3, 5, 6)
+    plans = [gar.gar_plan_create(3, n, "f32", "sum", 3), gar.gar_plan_create(5, n, "f32", "sum", 4),
+             gar.gar_plan_create(6, n, "f32", "sum", 5)]
+    count = 300
+    rng = np.random.default_rng(3)
+    which = rng.integers(0, 3, count)
+    sizes = [Ps[w] * n for w in which]
+    offs = np.concatenate([[0], np.cumsum(sizes)])[:-1] + 1    # +1 element: misaligned base
+    data = torch.randn(int(offs[-1] + sizes[-1] + 8), device=DEV)
+    ref_in = data.cpu().numpy().copy()
+    es = 4
+    desc = gar.make_batch_desc(which, [data.data_ptr() + int(o) * es for o in offs],
+                               [data.data_ptr() + int(o) * es for o in offs])
+    gar.gar_allreduce_batched(plans, desc, count)
+    torch.cuda.synchronize()
+    got = data.cpu().numpy()
+    steps = (3, 4, 5)
+    for i in range(count):
+        P, o, S = Ps[which[i]], int(offs[i]), steps[which[i]]
+        xs = [ref_in[o + x * n: o + (x + 1) * n].copy() for x in range(P)]
+        want = G.allreduce(xs, S, "sum", "f32")
+        for x in range(P):
+            np.testing.assert_array_equal(got[o + x * n: o + (x + 1) * n].view(np.uint32),
+                                          want[x].view(np.uint32))
+
+
+# ---------------------------------------------------------------------------
+# Host-buffer entry point and argument handling on the device
+# ---------------------------------------------------------------------------
+
+@pytest.mark.parametrize("mode", ["fused", "step"])
+def test_host_buffers(mode):
+    P, n = 7, 70001
+    t = _np_inputs(P, n, "f32", seed=11)
+    host_in = t.clone().pin_memory()
+    host_out = torch.empty_like(host_in).pin_memory()
+    dev_store, _ = _padded_device(t)
+    plan = gar.gar_plan_create(P, n, "f32", "sum", 4)
+    rows_in = [host_in[x] for x in range(P)]
+    rows_out = [host_out[x] for x in range(P)]
+    gar.gar_allreduce_host(plan, rows_in, rows_out, dev_store, mode)
+    torch.cuda.synchronize()
+    want = G.allreduce(_to_host_list(t, "f32"), 4, "sum", "f32")
+    _assert_same(host_out, want, "f32", "host")
+
+
+def test_missing_workspace_is_an_error():
+    P, n = 7, 100
+    plan = gar.gar_plan_create(P, n, "f32", "sum", 3)
+    store, _ = _padded_device(torch.zeros(P, n))
+    import ctypes
+    ptrs = (ctypes.c_void_p * P)(*[store[x].data_ptr() for x in range(P)])
+    rc = gar._lib.gar_allreduce(plan.handle, ptrs, gar.GAR_STEP_FAITHFUL,
+                                ctypes.c_void_p(torch.cuda.current_stream().cuda_stream))
+    assert rc == -6

@@ -1,0 +1,262 @@
+"""Host-side checks of libgar's schedule builder against the CPU oracle (no GPU).
+
+* the library loads and exports every function include/gar.h declares;
+* per communication step: transmitted placements, partner offset and message bytes
+  equal the oracle's simulated messages;
+* the origin map and the fused program's result trees equal the oracle's;
+* the step-faithful op tables, executed on the CPU with the kernels' semantics (all
+  reads of a launch see the state before it), give the oracle's results bit for bit
+  and never write a block another op of the same launch reads;
+* argument errors return the documented codes.
+"""
+
+import os
+import re
+
+import numpy as np
+import pytest
+import torch
+
+from oracle import gar_oracle as G
+from paper_2004_09362_gb300 import gar
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+BUF_NONE, BUF_RANK, BUF_QP0, BUF_QP1, BUF_QS = range(5)
+
+
+def test_library_exports_every_declared_function():
+    with open(os.path.join(ROOT, "include", "gar.h")) as f:
+        hdr = f.read()
+    declared = set(re.findall(r"GAR_API\s+[\w\s\*]*?\b(gar_\w+)\s*\(", hdr))
+    assert declared, "no declarations found"
+    assert declared == set(gar.EXPORTS)
+    import ctypes
+    lib = ctypes.CDLL(gar.lib_path())
+    for name in declared:
+        assert hasattr(lib, name), name
+
+
+def test_jit_compiles_without_gpu():
+    gar.gar_selftest_compile()
+
+
+def _cases():
+    out = []
+    for P in list(range(1, 41)) + [63, 64, 65, 127, 128, 129]:
+        L = G.ceil_log2(P)
+        for S in range(L, 2 * L + 1):
+            out.append((P, S))
+    return out
+
+
+@pytest.mark.parametrize("P,S", _cases())
+def test_schedule_matches_oracle(P, S):
+    n = 3 * P + 1 if P > 1 else 5
+    for dtype in ("f32", "bf16"):
+        plan = gar.gar_plan_create(P, n, dtype, "sum", S)
+        info = plan.info()
+        run = G.simulate(P, n, S, dtype=dtype)
+        assert (info["L"], info["S"], info["r"], info["K"]) == (run.L, run.steps, run.r, run.K)
+        ws, per_step, S_lib = gar.gar_plan_bytes(plan)
+        assert S_lib == S
+        assert per_step == run.step_bytes()
+        for t, st in enumerate(run.log):
+            phase, partner, tx = gar.gar_plan_step(plan, t)
+            assert phase == (0 if st["phase"] == "reduce" else 1)
+            assert partner == (st["d"] if phase == 0 else -st["d"])
+            assert sorted(tx) == sorted(k[0] for k in st["tx"])
+        # origin map: rank x's block b comes from placement (x - b); its tree is copy o
+        origin = gar.gar_plan_origin(plan)
+        root_of = {key[1]: s for s, key in enumerate(run.after_reduction)}
+        for p in range(P):
+            key = run.out_key[p % P][0]       # rank p, block 0 -> placement p
+            assert key[0] == p
+            assert root_of[key[1]] == origin[p]
+        # fused program trees == the oracle's result trees
+        pairs, outs = gar.gar_plan_fused_program(plan)
+        memo = {}
+
+        def tree(v):
+            if v < P:
+                return v
+            if v not in memo:
+                a, b = pairs[v - P]
+                memo[v] = (tree(a), tree(b))
+            return memo[v]
+
+        assert len(outs) == run.K
+        for s in range(run.K):
+            assert tree(outs[s]) == run.exprs.tree(run.after_reduction[s][1])
+
+
+def _blocks(n, P):
+    return G.block_bounds(n, P)
+
+
+def _to_acc(a, dtype):
+    return a.astype(np.int32 if dtype == "i32" else np.float32)
+
+
+def _round_store(a, dtype):
+    if dtype == "bf16":
+        return torch.from_numpy(np.ascontiguousarray(a, np.float32)).to(torch.bfloat16).float().numpy()
+    return a
+
+
+def _op(op, a, b):
+    if op == "sum":
+        return a + b
+    return np.maximum(a, b) if op == "max" else np.minimum(a, b)
+
+
+def emulate_step_faithful(plan, xs, dtype, op):
+    """Executes the plan's step-faithful op table on the CPU.  Rank buffers hold the
+    element type (bf16 values kept as float32 after rounding), workspace the
+    accumulation type.  Returns (outputs, per-launch recv element counts)."""
+    P = len(xs)
+    n = len(xs[0])
+    bounds = _blocks(n, P)
+    acc_dt = np.int32 if dtype == "i32" else np.float32
+    bufs = {BUF_RANK: [x.copy() for x in xs],
+            BUF_QP0: [np.zeros(n, acc_dt) for _ in range(P)],
+            BUF_QP1: [np.zeros(n, acc_dt) for _ in range(P)],
+            BUF_QS: [np.zeros(n, acc_dt) for _ in range(P)]}
+    ops, partners = gar.gar_plan_step_ops(plan)
+    for l, partner in enumerate(partners):
+        lops = ops[ops[:, 0] == l]
+        writes, reads, written = [], set(), {}
+        for (_l, recv_place, dst_place, recv_buf, o0b, o0o, o1b, o1o) in lops:
+            for x in range(P):
+                b = (x - dst_place) % P
+                lo, hi = bounds[b]
+                recv = None
+                if recv_place >= 0:
+                    src = (x + partner) % P
+                    assert (src - recv_place) % P == b      # same block at the partner
+                    recv = _to_acc(bufs[recv_buf][src][lo:hi], dtype)
+                    reads.add((recv_buf, src, b))
+                for (ob, oo) in ((o0b, o0o), (o1b, o1o)):
+                    if ob == BUF_NONE:
+                        continue
+                    if oo != BUF_NONE:
+                        own = _to_acc(bufs[oo][x][lo:hi], dtype)
+                        if oo != ob:
+                            reads.add((oo, x, b))
+                        val = own if recv is None else _op(op, own, recv)
+                    else:
+                        val = recv
+                    key = (ob, x, b)
+                    assert key not in written, "two ops write one block in a launch"
+                    written[key] = True
+                    writes.append((ob, x, lo, hi, val))
+        assert not (reads & set(written)), "a launch writes a block another op reads"
+        for (ob, x, lo, hi, val) in writes:
+            if ob == BUF_RANK:
+                bufs[BUF_RANK][x][lo:hi] = _round_store(val, dtype).astype(xs[0].dtype)
+            else:
+                bufs[ob][x][lo:hi] = val
+    return bufs[BUF_RANK]
+
+
+@pytest.mark.parametrize("P", list(range(1, 18)) + [24, 31, 33])
+def test_step_faithful_tables_reproduce_oracle(P):
+    rng = np.random.default_rng(P)
+    L = G.ceil_log2(P)
+    for n in sorted({max(P - 1, 1), 2 * P + 3}):
+        for dtype in ("f32", "i32", "bf16"):
+            if dtype == "i32":
+                xs = [rng.integers(-1000, 1001, n).astype(np.int32) for _ in range(P)]
+            else:
+                xs = [(rng.standard_normal(n) * np.exp2(rng.integers(-10, 11, n))).astype(np.float32)
+                      for _ in range(P)]
+                if dtype == "bf16":
+                    xs = [G.round_to_bf16(v) for v in xs]
+            for S in range(L, 2 * L + 1):
+                plan = gar.gar_plan_create(P, n, dtype, "sum", S)
+                got = emulate_step_faithful(plan, xs, dtype, "sum")
+                want = G.allreduce(xs, S, "sum", dtype)
+                for x in range(P):
+                    np.testing.assert_array_equal(got[x].view(np.uint32), want[x].view(np.uint32))
+
+
+def emulate_fused(plan, xs, op):
+    P = len(xs)
+    n = len(xs[0])
+    pairs, outs = gar.gar_plan_fused_program(plan)
+    origin = gar.gar_plan_origin(plan)
+    res = [np.empty_like(x) for x in xs]
+    for b, (lo, hi) in enumerate(_blocks(n, P)):
+        vals = [xs[(b + j) % P][lo:hi] for j in range(P)]
+        for (a, c) in pairs:
+            vals.append(_op(op, vals[a], vals[c]))
+        for p in range(P):
+            res[(b + p) % P][lo:hi] = vals[outs[origin[p]]]
+    return res
+
+
+@pytest.mark.parametrize("P", list(range(1, 20)) + [24, 40, 127])
+def test_fused_program_reproduces_oracle(P):
+    rng = np.random.default_rng(1000 + P)
+    L = G.ceil_log2(P)
+    n = 2 * P + 5
+    xs = [(rng.standard_normal(n) * np.exp2(rng.integers(-10, 11, n))).astype(np.float32)
+          for _ in range(P)]
+    for S in range(L, 2 * L + 1):
+        for op in ("sum", "max"):
+            plan = gar.gar_plan_create(P, n, "f32", op, S)
+            got = emulate_fused(plan, xs, op)
+            want = G.allreduce(xs, S, op, "f32")
+            for x in range(P):
+                np.testing.assert_array_equal(got[x].view(np.uint32), want[x].view(np.uint32))
+
+
+def test_workspace_sizes():
+    # bandwidth-optimal fp32/int32 runs in place
+    for P in (2, 5, 24, 127):
+        for dt in ("f32", "i32"):
+            ws, _, _ = gar.gar_plan_bytes(gar.gar_plan_create(P, 1000, dt, "sum", gar.GAR_STEPS_BO))
+            assert ws == 0
+    # bf16 keeps fp32 partials in one slice; other step counts need ping-pong (+ q*)
+    ws, _, _ = gar.gar_plan_bytes(gar.gar_plan_create(5, 1000, "bf16", "sum", gar.GAR_STEPS_BO))
+    assert ws == 5 * 1024 * 4
+    ws, _, _ = gar.gar_plan_bytes(gar.gar_plan_create(8, 1000, "f32", "sum", gar.GAR_STEPS_LO))
+    assert ws == 2 * 8 * 1024 * 4          # P = 2^k: q* never separates from q'
+    ws, _, _ = gar.gar_plan_bytes(gar.gar_plan_create(7, 1000, "f32", "sum", gar.GAR_STEPS_LO))
+    assert ws == 3 * 7 * 1024 * 4
+
+
+def test_argument_errors():
+    with pytest.raises(gar.GarError) as e:
+        gar.gar_plan_create(0, 10)
+    assert e.value.code == -1
+    with pytest.raises(gar.GarError):
+        gar.gar_plan_create(gar.GAR_MAX_P + 1, 10)
+    with pytest.raises(gar.GarError):
+        gar.gar_plan_create(5, 10, steps=2)          # L = 3
+    with pytest.raises(gar.GarError):
+        gar.gar_plan_create(5, 10, steps=7)
+    with pytest.raises(gar.GarError):
+        gar.gar_plan_create(5, 10, dtype=7)
+    with pytest.raises(gar.GarError):
+        gar.gar_plan_create(5, 10, op=9)
+    plan = gar.gar_plan_create(5, 10)
+    with pytest.raises(gar.GarError) as e:
+        gar.gar_allreduce(plan, [16 * (k + 1) for k in range(4)] + [16 * 3], "fused", stream=0)
+    assert e.value.code == -1
+    with pytest.raises(gar.GarError) as e:
+        gar.gar_allreduce(plan, [16 * (k + 1) + 4 for k in range(5)], "fused", stream=0)
+    assert e.value.code == -3
+    with pytest.raises(gar.GarError):
+        gar.gar_plan_step(plan, 99)
+    assert gar.gar_strerror(-3).startswith("buffer")
+    # P = 1 and n = 0 are accepted no-ops (no GPU work is launched)
+    gar.gar_allreduce(gar.gar_plan_create(1, 10), [64], "fused", stream=0)
+    gar.gar_allreduce(gar.gar_plan_create(4, 0), [64, 128, 192, 256], "fused", stream=0)
+
+
+def test_generated_source_compiles_for_config_shapes():
+    for (P, n, dt, S) in [(24, 16777216, "f32", 10), (127, 4194304, "bf16", 7), (127, 4194304, "bf16", 14),
+                          (8, 262144, "f32", 4), (5, 1024, "i32", 3)]:
+        plan = gar.gar_plan_create(P, n, dt, "sum", S)
+        gar.gar_plan_compile(plan, "fused")
+        assert plan.info()["fused_width"] >= 1
