@@ -130,6 +130,21 @@ class ClockSampler:
 # Timing helpers
 # ---------------------------------------------------------------------------
 
+def max_over_ranks(ms: float, dist, device) -> float:
+    """The slowest rank's time (ms); identity without a process group."""
+    if dist is None:
+        return ms
+    import torch
+    t = torch.tensor([float(ms)], dtype=torch.float64, device=device)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
+def job_gbs(bytes_per_replica: int, world: int, ms: float) -> float:
+    """Whole-job throughput: every replica's bytes over the slowest replica's time."""
+    return bytes_per_replica * world / (ms * 1e-3) / 1e9
+
+
 def _time_loop(fn, steps, warmup, stream, flush=None):
     """Runs fn() warmup times, then times `steps` calls with CUDA events on `stream`
     (synchronised on both sides).  With `flush`, L2 is flushed before every call and
@@ -182,12 +197,11 @@ def _alg_bytes(P, n, dtype):
 def _step_dram_bytes(gar, plan, P, n, dtype):
     """DRAM bytes one step-faithful Allreduce moves under the kernels' access pattern:
     per block op and rank, the partner read, the own reads and the writes."""
-    from oracle import gar_oracle  # block sizes only
     ops, _partners = gar.gar_plan_step_ops(plan)
     es = {"f32": 4, "bf16": 2, "i32": 4}[dtype]
     acc = 4
-    bounds = gar_oracle.block_bounds(n, P)
-    sizes = [hi - lo for (lo, hi) in bounds]
+    q, rem = divmod(n, P)
+    sizes = [q + (1 if b < rem else 0) for b in range(P)]
     tot = 0
     for (_l, recv_place, dst, recv_buf, o0b, o0o, o1b, o1o) in ops:
         for x in range(P):
@@ -246,13 +260,9 @@ def run_ours(args):
         torch.cuda.synchronize()
     if dist is not None:
         dist.barrier()
-    ms = start.elapsed_time(end) / args.steps
-    if dist is not None:
-        t = torch.tensor([ms], device="cuda")
-        dist.all_reduce(t, op=dist.ReduceOp.MAX)
-        ms = float(t.item())
+    ms = max_over_ranks(start.elapsed_time(end) / args.steps, dist, "cuda")
     bytes_step = _alg_bytes(P, n, wl.dtype)
-    value = bytes_step * ws / (ms * 1e-3) / 1e9
+    value = job_gbs(bytes_step, ws, ms)
     clocks = clk.summary()
     kernel_gbs = bytes_step / (ms * 1e-3) / 1e9
 
@@ -289,17 +299,26 @@ def run_ours(args):
 
 
 def _committed_traffic():
-    """dram bytes per launch of the headline fused kernel from the committed ncu summary
-    (profiles/fused_p24_64mib_f32.txt), or None when absent."""
+    """DRAM bytes per launch of the headline fused kernel from the committed ncu summary
+    (profiles/fused_p24_64mib_f32.txt), or None when absent or when the kernel generator
+    (csrc/codegen.cpp) has changed since the counters were taken."""
+    import hashlib
     path = os.path.join(ROOT, "profiles", "fused_p24_64mib_f32.txt")
+    src = os.path.join(ROOT, "paper_2004_09362_gb300", "csrc", "codegen.cpp")
     try:
+        with open(src, "rb") as f:
+            sha = hashlib.sha1(f.read()).hexdigest()[:12]
+        fields = {}
         with open(path) as f:
             for line in f:
-                if line.startswith("dram_bytes_per_launch:"):
-                    return int(line.split(":", 1)[1].strip().split()[0])
+                if ":" in line and not line.startswith(" "):
+                    k, v = line.split(":", 1)
+                    fields[k.strip()] = v.strip()
+        if fields.get("codegen_sha1") != sha:
+            return None
+        return int(fields["dram_bytes_per_launch"].split()[0])
     except Exception:
-        pass
-    return None
+        return None
 
 
 def _e2e(gar, plan, inp, P, n, args, stream, dist):
@@ -317,14 +336,10 @@ def _e2e(gar, plan, inp, P, n, args, stream, dist):
         gar.gar_allreduce_host(plan, hp_in, hp_out, dp, "fused", stream)
 
     steps = max(1, min(args.steps, 10))
-    ms = _time_loop(step, steps, max(1, min(args.warmup, 3)), stream)
-    if dist is not None:
-        t = torch.tensor([ms], device="cuda")
-        dist.all_reduce(t, op=dist.ReduceOp.MAX)
-        ms = float(t.item())
+    ms = max_over_ranks(_time_loop(step, steps, 3, stream), dist, "cuda")
     ws = dist.get_world_size() if dist is not None else 1
     bytes_step = _alg_bytes(P, n, "f32")
-    return {"value": round(bytes_step * ws / (ms * 1e-3) / 1e9, 2), "unit": "GB/s",
+    return {"value": round(job_gbs(bytes_step, ws, ms), 2), "unit": "GB/s",
             "ms_per_step": round(ms, 4), "h2d_bytes_per_step": P * n * 4,
             "d2h_bytes_per_step": P * n * 4, "steps": steps,
             "path": "gar_allreduce_host: P cudaMemcpyAsync H2D from pinned memory, fused kernel, P D2H"}
@@ -450,23 +465,27 @@ def _oracle_time(P, n, S, dtype="f32", seed=1237):
 
 def cpu_baseline_sample(target_s=10.0):
     """The oracle as it stands (single-threaded numpy) on the headline workload's shape
-    (P = 24, S = 10, fp32 sum) with fewer elements per rank, sized to take about
-    target_s seconds.  Reported in the headline's unit (algorithmic GB/s)."""
+    (P = 24, S = 10, fp32 sum) with at most the headline's elements per rank, repeated
+    until about target_s seconds of CPU work.  Reported in the headline's unit
+    (algorithmic GB/s per Allreduce)."""
     P, S = 24, 10
+    n_max = 16777216
     n = 24 * 4096
     dt = _oracle_time(P, n, S)
-    while dt < target_s / 8 and n < 24 * 2 ** 20:
+    while dt < target_s / 10 and n * 2 <= n_max:
         n *= 2
         dt = _oracle_time(P, n, S)
-    if dt < target_s / 2 and n < 24 * 2 ** 21:
-        n = int(n * min(8.0, target_s / max(dt, 1e-3)) // 24 * 24)
-        dt = _oracle_time(P, n, S)
+    reps, total = 1, dt
+    while total < target_s:
+        total += _oracle_time(P, n, S)
+        reps += 1
+    sec = total / reps
     cores, model = _cpu_info()
-    gbs = _alg_bytes(P, n, "f32") / dt / 1e9
+    gbs = _alg_bytes(P, n, "f32") / sec / 1e9
     return {"value": round(gbs, 4), "unit": "GB/s", "cores": 1, "host_cores": cores,
-            "cpu_model": model, "kind": "oracle", "seconds": round(dt, 2),
+            "cpu_model": model, "kind": "oracle", "seconds": round(total, 2),
             "sample": f"P=24, S=10 (bandwidth-optimal), fp32 sum, n={n} elements per rank "
-                      f"(headline has 16777216), one Allreduce"}
+                      f"(headline has {n_max}), {reps} Allreduce(s), mean time"}
 
 
 def run_reference(args):
@@ -479,7 +498,7 @@ def run_reference(args):
     per_step = max(1.0, min(20.0, budget / max(1, args.steps + args.warmup)))
     n = 24 * 4096
     dt = _oracle_time(P, n, S)
-    while dt < per_step / 2 and n < 24 * 2 ** 21:
+    while dt < per_step / 2 and n * 2 <= 16777216:
         n *= 2
         dt = _oracle_time(P, n, S)
     for _ in range(args.warmup):
