@@ -202,6 +202,26 @@ GAR_API int gar_last_step_bytes(const gar_plan *plan, uint64_t *per_step);
 GAR_API const char *gar_strerror(int status);
 GAR_API const char *gar_last_error(void);
 
+/* Step-faithful Allreduce that allocates no device memory.  The paper has no
+ * counterpart; this entry point serves callers that cannot call cudaMalloc when they
+ * run an Allreduce, e.g. code whose device memory is all owned by a caching
+ * allocator or by another runtime.  Same result as gar_allreduce(plan, rank_buffers,
+ * GAR_STEP_FAITHFUL, stream), but the workspace is a fixed file-scope device array of
+ * GAR_NOALLOC_SCRATCH_BYTES, reserved on every GPU that loads the library until the
+ * process exits, and the block ops travel in the kernel parameters; the plan's workspace
+ * and device tables are not used, no bytes are recorded, and no cudaMalloc, cudaFree or
+ * other allocating call is made.
+ * Limits: P <= GAR_NOALLOC_MAX_P and a workspace (gar_plan_bytes) of at most
+ * GAR_NOALLOC_SCRATCH_BYTES; larger plans return GAR_EINVAL with the sizes in
+ * gar_last_error().  The first call on a device looks up the array's device address
+ * (cudaGetSymbolAddress) with that device current; make that first call before any
+ * stream capture.  All calls share the one array and leave their partial results in it:
+ * calls whose work overlaps on the GPU (other streams, other host threads) race, so
+ * order them on one stream.  rank_buffers: as for gar_allreduce. */
+#define GAR_NOALLOC_SCRATCH_BYTES (64u << 20)
+#define GAR_NOALLOC_MAX_P 64
+GAR_API int gar_allreduce_noalloc(gar_plan *plan, void *const *rank_buffers, gar_stream_t stream);
+
 /* Library self-test for build checks: generates and compiles (host-only, no GPU) the
  * fused kernels of a few plans.  Returns GAR_OK or GAR_EJIT. */
 GAR_API int gar_selftest_compile(void);

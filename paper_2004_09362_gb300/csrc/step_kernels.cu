@@ -12,6 +12,8 @@
 #include <cuda_runtime.h>
 
 #include <cstdint>
+#include <mutex>
+#include <string>
 
 #include "gar_internal.hpp"
 
@@ -270,3 +272,231 @@ int launch_step(const gar_plan &pl, const Launch &ln, int launch_index, void *co
 }
 
 }  // namespace gar
+
+// ---------------------------------------------------------------------------
+// Step-faithful Allreduce without device allocation (gar_allreduce_noalloc).
+//
+// For callers that must not allocate device memory at call time -- code running
+// under a caching allocator that owns all of the GPU's memory, or a host runtime with
+// no allocator hook -- the workspace lives in one file-scope device array of fixed
+// size instead of a caller-supplied buffer, and each launch receives its block ops by
+// value in the kernel parameters instead of from a device table.  No cudaMalloc,
+// cudaFree or memset is issued.  The array is reserved on every device that loads
+// this library and stays reserved until the process exits.  Nothing in it needs to
+// start at zero: the schedule writes every workspace slot before it reads it.  All
+// calls share the array, so two calls whose work overlaps on the GPU race.
+// ---------------------------------------------------------------------------
+
+static __device__ __align__(256) unsigned char g_noalloc_scratch[GAR_NOALLOC_SCRATCH_BYTES];
+
+namespace gar {
+namespace {
+
+constexpr int kNoAllocMaxOps = 2 * GAR_NOALLOC_MAX_P;  // |transmit set| + K <= 2P per launch
+
+struct NoAllocArgs {
+  void *rank[GAR_NOALLOC_MAX_P];
+  void *ws[NUM_WS_BUFS];
+  StepOp ops[kNoAllocMaxOps];
+  uint64_t q, rem, n_pad;
+  int P, partner, nops, nchunks;
+};
+
+template <typename A>
+__device__ __forceinline__ void *na_buf_ptr(const NoAllocArgs &a, uint8_t buf, int rank) {
+  if (buf == BUF_RANK) return a.rank[rank];
+  if (buf == BUF_NONE) return nullptr;
+  return static_cast<char *>(a.ws[buf - BUF_QP0]) + (uint64_t)rank * a.n_pad * sizeof(A);
+}
+
+// Same block-op semantics as step_kernel (one CTA per op x rank x chunk), with the ops
+// read from the parameter block and no byte counting.
+template <typename T, int OP>
+__global__ void __launch_bounds__(kThreads) step_kernel_noalloc(const __grid_constant__ NoAllocArgs a) {
+  using A = typename AccOf<T>::type;
+  uint64_t bid = blockIdx.x;
+  const int chunk = (int)(bid % (uint64_t)a.nchunks);
+  bid /= (uint64_t)a.nchunks;
+  const int x = (int)(bid % (uint64_t)a.P);
+  const int oi = (int)(bid / (uint64_t)a.P);
+  if (oi >= a.nops) return;
+  const StepOp op = a.ops[oi];
+  const int b = ((x - (int)op.dst_place) % a.P + a.P) % a.P;
+  const uint64_t bstart = (uint64_t)b * a.q + ((uint64_t)b < a.rem ? (uint64_t)b : a.rem);
+  const uint64_t blen = a.q + ((uint64_t)b < a.rem ? 1 : 0);
+  const uint64_t c0 = (uint64_t)chunk * kChunk;
+  if (c0 >= blen) return;
+  const uint64_t lo = bstart + c0;
+  const uint64_t hi = bstart + (blen < c0 + kChunk ? blen : c0 + kChunk);
+  const bool has_recv = op.recv_place >= 0;
+  const int partner = ((x + a.partner) % a.P + a.P) % a.P;
+  const void *recv = has_recv ? na_buf_ptr<A>(a, op.recv_buf, partner) : nullptr;
+  void *out0 = na_buf_ptr<A>(a, op.out0_buf, x);
+  const void *own0 = na_buf_ptr<A>(a, op.out0_own, x);
+  void *out1 = na_buf_ptr<A>(a, op.out1_buf, x);
+  const void *own1 = na_buf_ptr<A>(a, op.out1_own, x);
+
+  auto result = [&](const void *own, uint8_t own_buf, uint64_t e, A r) -> A {
+    if (!own) return r;
+    const A o = load1<T, A>(own_buf, own, e);
+    return has_recv ? combine<OP>(o, r) : o;
+  };
+  auto do1 = [&](uint64_t e) {
+    const A r = has_recv ? load1<T, A>(op.recv_buf, recv, e) : A(0);
+    const A o0 = result(own0, op.out0_own, e, r);
+    const A o1 = out1 ? result(own1, op.out1_own, e, r) : r;
+    store1<T, A>(op.out0_buf, out0, e, o0);
+    if (out1) store1<T, A>(op.out1_buf, out1, e, o1);
+  };
+  auto do4 = [&](uint64_t e) {
+    A r[4] = {A(0), A(0), A(0), A(0)};
+    if (has_recv) load4<T, A>(op.recv_buf, recv, e, r);
+    A o0[4], o1[4];
+#pragma unroll
+    for (int k = 0; k < 4; ++k) o0[k] = o1[k] = r[k];
+    if (own0) {
+      load4<T, A>(op.out0_own, own0, e, o0);
+      if (has_recv)
+#pragma unroll
+        for (int k = 0; k < 4; ++k) o0[k] = combine<OP>(o0[k], r[k]);
+    }
+    if (out1 && own1) {
+      load4<T, A>(op.out1_own, own1, e, o1);
+      if (has_recv)
+#pragma unroll
+        for (int k = 0; k < 4; ++k) o1[k] = combine<OP>(o1[k], r[k]);
+    }
+    store4<T, A>(op.out0_buf, out0, e, o0);
+    if (out1) store4<T, A>(op.out1_buf, out1, e, o1);
+  };
+  uint64_t va = (lo + 3) & ~uint64_t(3);
+  uint64_t vb = hi & ~uint64_t(3);
+  if (va > hi) va = hi;
+  if (vb < va) vb = va;
+  for (uint64_t e = lo + threadIdx.x; e < va; e += blockDim.x) do1(e);
+  for (uint64_t e = va + 4 * (uint64_t)threadIdx.x; e < vb; e += 4 * (uint64_t)blockDim.x) do4(e);
+  for (uint64_t e = vb + threadIdx.x; e < hi; e += blockDim.x) do1(e);
+}
+
+std::mutex g_noalloc_mu;
+void *g_noalloc_ptr[64] = {};
+
+// Device address of the scratch array on the current device.  The first call on a
+// device resolves it (with that device current) and caches it; later calls reuse it.
+int noalloc_scratch(void **out) {
+  int dev = -1;
+  cudaError_t e = cudaGetDevice(&dev);
+  if (e != cudaSuccess) return cuda_fail(e, "cudaGetDevice");
+  if (dev < 0 || dev >= 64) {
+    set_error("device ordinal out of range for the no-allocation scratch table");
+    return GAR_EINVAL;
+  }
+  std::lock_guard<std::mutex> lock(g_noalloc_mu);
+  if (g_noalloc_ptr[dev] == nullptr) {
+    void *p = nullptr;
+    e = cudaGetSymbolAddress(&p, g_noalloc_scratch);
+    if (e != cudaSuccess) return cuda_fail(e, "cudaGetSymbolAddress(no-allocation scratch)");
+    g_noalloc_ptr[dev] = p;
+  }
+  *out = g_noalloc_ptr[dev];
+  return GAR_OK;
+}
+
+template <typename T, int OP>
+int noalloc_launch(const gar_plan &pl, const Launch &ln, void *const *rank, void *scratch,
+                   gar_stream_t stream) {
+  NoAllocArgs a{};
+  for (int x = 0; x < pl.P; ++x) a.rank[x] = rank[x];
+  int slot = 0;
+  for (int k = 0; k < NUM_WS_BUFS; ++k) {
+    a.ws[k] = pl.ws_used[k] ? static_cast<char *>(scratch) +
+                                  (size_t)(slot++) * pl.P * pl.n_pad * acc_size(pl.dtype)
+                            : nullptr;
+  }
+  for (int k = 0; k < ln.nops; ++k) a.ops[k] = pl.ops[ln.first_op + k];
+  a.q = pl.q;
+  a.rem = pl.rem;
+  a.n_pad = pl.n_pad;
+  a.P = pl.P;
+  a.partner = ln.partner;
+  a.nops = ln.nops;
+  const uint64_t maxblk = pl.q + (pl.rem ? 1 : 0);
+  a.nchunks = (int)((maxblk + kChunk - 1) / kChunk);
+  if (a.nchunks == 0 || ln.nops == 0) return GAR_OK;
+  const uint64_t grid = (uint64_t)a.nchunks * (uint64_t)pl.P * (uint64_t)ln.nops;
+  if (grid > 0x7fffffffull) {
+    set_error("no-allocation step launch grid too large");
+    return GAR_EINVAL;
+  }
+  step_kernel_noalloc<T, OP><<<(unsigned)grid, kThreads, 0, (cudaStream_t)stream>>>(a);
+  cudaError_t e = cudaGetLastError();
+  if (e != cudaSuccess) return cuda_fail(e, "no-allocation step kernel launch");
+  return GAR_OK;
+}
+
+template <typename T>
+int noalloc_launch_op(const gar_plan &pl, const Launch &ln, void *const *rank, void *scratch,
+                      gar_stream_t s) {
+  switch (pl.op) {
+    case GAR_SUM: return noalloc_launch<T, GAR_SUM>(pl, ln, rank, scratch, s);
+    case GAR_MAX: return noalloc_launch<T, GAR_MAX>(pl, ln, rank, scratch, s);
+    case GAR_MIN: return noalloc_launch<T, GAR_MIN>(pl, ln, rank, scratch, s);
+  }
+  return GAR_EINVAL;
+}
+
+}  // namespace
+}  // namespace gar
+
+extern "C" int gar_allreduce_noalloc(gar_plan *pl, void *const *rank_buffers, gar_stream_t stream) {
+  using namespace gar;
+  if (pl == nullptr || rank_buffers == nullptr) {
+    set_error("null plan or rank buffer array");
+    return GAR_EINVAL;
+  }
+  if (pl->P > GAR_NOALLOC_MAX_P) {
+    set_error("gar_allreduce_noalloc supports P <= " + std::to_string(GAR_NOALLOC_MAX_P) +
+              ", plan has P=" + std::to_string(pl->P));
+    return GAR_EINVAL;
+  }
+  if (pl->ws_bytes > (size_t)GAR_NOALLOC_SCRATCH_BYTES) {
+    set_error("gar_allreduce_noalloc: plan needs " + std::to_string(pl->ws_bytes) +
+              " bytes of workspace, the fixed scratch array holds " +
+              std::to_string((size_t)GAR_NOALLOC_SCRATCH_BYTES));
+    return GAR_EINVAL;
+  }
+  for (int x = 0; x < pl->P; ++x) {
+    if (rank_buffers[x] == nullptr) {
+      set_error("null rank buffer " + std::to_string(x));
+      return GAR_EINVAL;
+    }
+    if (reinterpret_cast<uintptr_t>(rank_buffers[x]) % 16 != 0) {
+      set_error("rank buffer " + std::to_string(x) + " is not 16-byte aligned");
+      return GAR_EALIGN;
+    }
+    for (int y = 0; y < x; ++y)
+      if (rank_buffers[y] == rank_buffers[x]) {
+        set_error("two ranks share one buffer");
+        return GAR_EINVAL;
+      }
+  }
+  for (const Launch &ln : pl->launches)
+    if (ln.nops > kNoAllocMaxOps) {
+      set_error("gar_allreduce_noalloc: a launch has more block ops than the parameter block holds");
+      return GAR_EINVAL;
+    }
+  if (pl->n == 0 || pl->P == 1) return GAR_OK;
+  void *scratch = nullptr;
+  int rc = noalloc_scratch(&scratch);
+  if (rc) return rc;
+  for (const Launch &ln : pl->launches) {
+    switch (pl->dtype) {
+      case GAR_F32: rc = noalloc_launch_op<float>(*pl, ln, rank_buffers, scratch, stream); break;
+      case GAR_BF16: rc = noalloc_launch_op<__nv_bfloat16>(*pl, ln, rank_buffers, scratch, stream); break;
+      case GAR_I32: rc = noalloc_launch_op<int>(*pl, ln, rank_buffers, scratch, stream); break;
+      default: rc = GAR_EINVAL;
+    }
+    if (rc) return rc;
+  }
+  return GAR_OK;
+}

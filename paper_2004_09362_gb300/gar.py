@@ -34,7 +34,7 @@ EXPORTS = (
     "gar_plan_step", "gar_plan_origin", "gar_plan_fused_program", "gar_plan_step_ops",
     "gar_plan_set_workspace", "gar_plan_compile", "gar_plan_prepare", "gar_allreduce",
     "gar_allreduce_host", "gar_allreduce_batched", "gar_last_step_bytes", "gar_strerror",
-    "gar_last_error", "gar_selftest_compile",
+    "gar_last_error", "gar_selftest_compile", "gar_allreduce_noalloc",
 )
 
 
@@ -76,6 +76,7 @@ def _load():
         "gar_strerror": (ctypes.c_char_p, [i32]),
         "gar_last_error": (ctypes.c_char_p, []),
         "gar_selftest_compile": (i32, []),
+        "gar_allreduce_noalloc": (i32, [vp, P_(vp), vp]),
     }
     for name, (res, args) in sig.items():
         fn = getattr(lib, name)
@@ -304,6 +305,12 @@ def gar_allreduce_batched(plans: Sequence[Plan], desc, count: int, stream=None) 
     dptr = desc if isinstance(desc, int) else desc.data_ptr()
     _check(_lib.gar_allreduce_batched(arr, len(plans), ctypes.c_void_p(dptr), int(count),
                                       _stream_handle(stream)), "gar_allreduce_batched")
+
+
+def gar_allreduce_noalloc(plan: Plan, rank_buffers, stream=None) -> None:
+    ptrs = _ptr_array(rank_pointers(rank_buffers))
+    _check(_lib.gar_allreduce_noalloc(plan.handle, ptrs, _stream_handle(stream)),
+           "gar_allreduce_noalloc")
 
 
 def gar_last_step_bytes(plan: Plan) -> list[int]:
