@@ -342,7 +342,7 @@ def _e2e(gar, plan, inp, P, n, args, stream, dist):
     return {"value": round(job_gbs(bytes_step, ws, ms), 2), "unit": "GB/s",
             "ms_per_step": round(ms, 4), "h2d_bytes_per_step": P * n * 4,
             "d2h_bytes_per_step": P * n * 4, "steps": steps,
-            "path": "gar_allreduce_host: P cudaMemcpyAsync H2D from pinned memory, fused kernel, P D2H"}
+            "path": "gar_allreduce_host on pinned host buffers: the fused kernel reads the P inputs from and writes the P results to host memory over NVLink-C2C (no staging copies)"}
 
 
 def measure_rows(gar, gar_inputs, stream, hbm_peak):

@@ -171,9 +171,16 @@ GAR_API int gar_plan_prepare(gar_plan *plan, int mode);
  * same tree). */
 GAR_API int gar_allreduce(gar_plan *plan, void *const *rank_buffers, int mode, gar_stream_t stream);
 
-/* Host-buffer Allreduce: copies host_in[x] (P host pointers, pinned memory gives full
- * speed) to dev_bufs[x], runs gar_allreduce on dev_bufs, and copies the results to
- * host_out[x] (may equal host_in).  Each copy is one cudaMemcpyAsync on `stream`.
+/* Host-buffer Allreduce: the P inputs host_in[x] are in host memory and the P results
+ * go to host memory host_out[x] (host_out[x] may equal host_in[x], or another rank's
+ * host_in; other overlaps are undefined).
+ * GAR_FUSED with 16-byte-aligned host buffers that the GPU can address directly (pinned
+ * or registered memory, or any host memory on a system with coherent host access such
+ * as NVLink-C2C): one fused kernel reads the inputs from and writes the results to host
+ * memory itself; dev_bufs is not used and may be NULL.  Otherwise the inputs are copied
+ * (cudaMemcpyAsync per rank and element chunk) to dev_bufs -- P device buffers as for
+ * gar_allreduce -- reduced there, and copied back; in fused mode the chunks pipeline
+ * over internal streams that are forked from and joined back into `stream`.
  * Returns after enqueueing; synchronize the stream before reading host_out. */
 GAR_API int gar_allreduce_host(gar_plan *plan, const void *const *host_in, void *const *host_out,
                        void *const *dev_bufs, int mode, gar_stream_t stream);

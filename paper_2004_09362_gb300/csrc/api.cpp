@@ -2,6 +2,7 @@
 #include <cuda_runtime.h>
 
 #include <algorithm>
+#include <cstdlib>
 #include <cstring>
 #include <new>
 #include <string>
@@ -121,21 +122,126 @@ int grid_for(const JitKernel *k, uint64_t work_items) {
   cudaGetDevice(&dev);
   cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
   if (sms <= 0) sms = 1;
+  // One work item per thread: with many more CTAs than fit at once the block scheduler
+  // keeps every SM full and each thread's loads are in flight together (a persistent
+  // grid-stride loop serialises a thread's iterations and ran 6% slower on GB300).
+  // GAR_TUNE_GRID_WAVES caps the grid at that many waves of resident CTAs (launch-shape
+  // sweeps only); the kernels' grid-stride loops cover any remainder.
   const uint64_t need = (work_items + k->threads - 1) / k->threads;
-  const uint64_t wave = (uint64_t)sms * (uint64_t)std::max(1, k->blocks_per_sm);
-  return (int)std::max<uint64_t>(1, std::min<uint64_t>(need, wave));
+  uint64_t cap = 0x7fffffffull;
+  const char *wv = std::getenv("GAR_TUNE_GRID_WAVES");
+  if (wv && std::atoi(wv) > 0)
+    cap = (uint64_t)sms * (uint64_t)std::max(1, k->blocks_per_sm) * (uint64_t)std::atoi(wv);
+  return (int)std::max<uint64_t>(1, std::min<uint64_t>(need, cap));
+}
+
+// One fused launch over element positions [e_lo, e_hi) (e_lo a multiple of the
+// kernel's vector width).  The parameter block is the generated kernel's gar_args:
+// P input pointers, P output pointers, e_lo, e_hi.
+int launch_fused_range(gar_plan *pl, const void *const *in, void *const *out, uint64_t e_lo,
+                       uint64_t e_hi, gar_stream_t stream) {
+  if (e_hi <= e_lo) return GAR_OK;
+  const size_t pb = 8 * (size_t)pl->P;
+  std::vector<unsigned char> args(2 * pb + 16);
+  std::memcpy(args.data(), in, pb);
+  std::memcpy(args.data() + pb, out, pb);
+  std::memcpy(args.data() + 2 * pb, &e_lo, 8);
+  std::memcpy(args.data() + 2 * pb + 8, &e_hi, 8);
+  void *kargs[] = {args.data()};
+  const uint64_t items = (e_hi - e_lo) / pl->fused->width + 1;
+  const int grid = grid_for(pl->fused, items);
+  cudaError_t e = cudaLaunchKernel((const void *)pl->fused->kernel, dim3(grid),
+                                   dim3(pl->fused->threads), kargs, 0, (cudaStream_t)stream);
+  if (e != cudaSuccess) return cuda_fail(e, "fused kernel launch");
+  return GAR_OK;
 }
 
 int run_fused(gar_plan *pl, void *const *rank, gar_stream_t stream) {
   int rc = prepare_fused(pl);
   if (rc) return rc;
-  std::vector<void *> args(rank, rank + pl->P);
-  void *kargs[] = {args.data()};
-  const uint64_t items = pl->n / pl->fused->width + 1;
-  const int grid = grid_for(pl->fused, items);
-  cudaError_t e = cudaLaunchKernel((const void *)pl->fused->kernel, dim3(grid),
-                                   dim3(pl->fused->threads), kargs, 0, (cudaStream_t)stream);
-  if (e != cudaSuccess) return cuda_fail(e, "fused kernel launch");
+  return launch_fused_range(pl, rank, rank, 0, pl->n, stream);
+}
+
+// True when every pointer is host memory the GPU can read and write directly (pinned or
+// registered memory, or any host memory on a system with coherent access such as
+// NVLink-C2C), so a kernel can use it without staging copies.
+bool device_accessible_host(const void *const *ptrs, int count) {
+  int dev = 0, pageable = 0;
+  cudaGetDevice(&dev);
+  cudaDeviceGetAttribute(&pageable, cudaDevAttrPageableMemoryAccess, dev);
+  for (int x = 0; x < count; ++x) {
+    cudaPointerAttributes at{};
+    if (cudaPointerGetAttributes(&at, ptrs[x]) != cudaSuccess) {
+      cudaGetLastError();
+      return false;
+    }
+    const bool pinned = at.type == cudaMemoryTypeHost && at.devicePointer == ptrs[x];
+    const bool pageable_ok = at.type == cudaMemoryTypeUnregistered && pageable;
+    if (!pinned && !pageable_ok) return false;
+  }
+  return true;
+}
+
+// Internal streams and events of the pipelined host-buffer path (created once).
+int prepare_host_pipeline(gar_plan *pl) {
+  if (pl->hp_ready) return GAR_OK;
+  cudaError_t e = cudaSuccess;
+  for (int k = 0; k < 3 && e == cudaSuccess; ++k)
+    e = cudaStreamCreateWithFlags((cudaStream_t *)&pl->hp_stream[k], cudaStreamNonBlocking);
+  for (int c = 0; c < GAR_HOST_CHUNKS_MAX && e == cudaSuccess; ++c) {
+    e = cudaEventCreateWithFlags((cudaEvent_t *)&pl->hp_h2d[c], cudaEventDisableTiming);
+    if (e == cudaSuccess) e = cudaEventCreateWithFlags((cudaEvent_t *)&pl->hp_krn[c], cudaEventDisableTiming);
+  }
+  if (e == cudaSuccess) e = cudaEventCreateWithFlags((cudaEvent_t *)&pl->hp_start, cudaEventDisableTiming);
+  if (e == cudaSuccess) e = cudaEventCreateWithFlags((cudaEvent_t *)&pl->hp_done, cudaEventDisableTiming);
+  if (e != cudaSuccess) return cuda_fail(e, "creating host-pipeline streams/events");
+  pl->hp_ready = true;
+  return GAR_OK;
+}
+
+// Fused Allreduce of host buffers, pipelined over element chunks: the copy of chunk c
+// to the device, the kernel on chunk c and the copy of chunk c back run on three
+// streams, so both copy directions and the kernel overlap.  Every element position
+// depends only on the P contributions at that position, so chunks are independent.
+int run_host_pipelined(gar_plan *pl, const void *const *host_in, void *const *host_out,
+                       void *const *dev, gar_stream_t stream) {
+  int rc = prepare_fused(pl);
+  if (rc) return rc;
+  rc = prepare_host_pipeline(pl);
+  if (rc) return rc;
+  const size_t es = (size_t)elem_size(pl->dtype);
+  const uint64_t n = pl->n;
+  uint64_t chunk = (n + GAR_HOST_CHUNKS_MAX - 1) / GAR_HOST_CHUNKS_MAX;
+  chunk = std::max<uint64_t>(chunk, (uint64_t)1 << 16);
+  chunk = (chunk + 63) / 64 * 64;
+  const int nchunks = (int)((n + chunk - 1) / chunk);
+  cudaStream_t s_in = (cudaStream_t)pl->hp_stream[0], s_k = (cudaStream_t)pl->hp_stream[1],
+               s_out = (cudaStream_t)pl->hp_stream[2];
+  cudaError_t e = cudaEventRecord((cudaEvent_t)pl->hp_start, (cudaStream_t)stream);
+  for (int k = 0; k < 3 && e == cudaSuccess; ++k)
+    e = cudaStreamWaitEvent((cudaStream_t)pl->hp_stream[k], (cudaEvent_t)pl->hp_start, 0);
+  if (e != cudaSuccess) return cuda_fail(e, "host pipeline: fork");
+  for (int c = 0; c < nchunks; ++c) {
+    const uint64_t lo = (uint64_t)c * chunk, hi = std::min<uint64_t>(n, lo + chunk);
+    const size_t off = (size_t)lo * es, bytes = (size_t)(hi - lo) * es;
+    for (int x = 0; x < pl->P && e == cudaSuccess; ++x)
+      e = cudaMemcpyAsync(static_cast<char *>(dev[x]) + off, static_cast<const char *>(host_in[x]) + off,
+                          bytes, cudaMemcpyHostToDevice, s_in);
+    if (e == cudaSuccess) e = cudaEventRecord((cudaEvent_t)pl->hp_h2d[c], s_in);
+    if (e == cudaSuccess) e = cudaStreamWaitEvent(s_k, (cudaEvent_t)pl->hp_h2d[c], 0);
+    if (e != cudaSuccess) return cuda_fail(e, "host pipeline: host to device");
+    rc = launch_fused_range(pl, dev, dev, lo, hi, (gar_stream_t)s_k);
+    if (rc) return rc;
+    e = cudaEventRecord((cudaEvent_t)pl->hp_krn[c], s_k);
+    if (e == cudaSuccess) e = cudaStreamWaitEvent(s_out, (cudaEvent_t)pl->hp_krn[c], 0);
+    for (int x = 0; x < pl->P && e == cudaSuccess; ++x)
+      e = cudaMemcpyAsync(static_cast<char *>(host_out[x]) + off, static_cast<const char *>(dev[x]) + off,
+                          bytes, cudaMemcpyDeviceToHost, s_out);
+    if (e != cudaSuccess) return cuda_fail(e, "host pipeline: device to host");
+  }
+  e = cudaEventRecord((cudaEvent_t)pl->hp_done, s_out);
+  if (e == cudaSuccess) e = cudaStreamWaitEvent((cudaStream_t)stream, (cudaEvent_t)pl->hp_done, 0);
+  if (e != cudaSuccess) return cuda_fail(e, "host pipeline: join");
   return GAR_OK;
 }
 
@@ -218,6 +324,15 @@ void gar_plan_destroy(gar_plan *pl) {
   if (pl == nullptr) return;
   if (pl->d_ops) cudaFree(pl->d_ops);
   if (pl->d_step_bytes) cudaFree(pl->d_step_bytes);
+  if (pl->hp_ready) {
+    for (int k = 0; k < 3; ++k) cudaStreamDestroy((cudaStream_t)pl->hp_stream[k]);
+    for (int c = 0; c < GAR_HOST_CHUNKS_MAX; ++c) {
+      cudaEventDestroy((cudaEvent_t)pl->hp_h2d[c]);
+      cudaEventDestroy((cudaEvent_t)pl->hp_krn[c]);
+    }
+    cudaEventDestroy((cudaEvent_t)pl->hp_start);
+    cudaEventDestroy((cudaEvent_t)pl->hp_done);
+  }
   delete pl;
 }
 
@@ -351,14 +466,30 @@ int gar_allreduce_host(gar_plan *pl, const void *const *host_in, void *const *ho
     set_error("null host buffer array");
     return GAR_EINVAL;
   }
-  if (int rc = check_buffers(pl, dev_bufs)) return rc;
-  const size_t bytes = (size_t)pl->n * (size_t)elem_size(pl->dtype);
   for (int x = 0; x < pl->P; ++x) {
     if (host_in[x] == nullptr || host_out[x] == nullptr) {
       set_error("null host buffer");
       return GAR_EINVAL;
     }
   }
+  if (pl->n == 0) return GAR_OK;
+  const size_t bytes = (size_t)pl->n * (size_t)elem_size(pl->dtype);
+  if (mode == GAR_FUSED && pl->P > 1) {
+    bool aligned = true;
+    for (int x = 0; x < pl->P; ++x)
+      aligned = aligned && reinterpret_cast<uintptr_t>(host_in[x]) % 16 == 0 &&
+                reinterpret_cast<uintptr_t>(host_out[x]) % 16 == 0;
+    if (aligned && device_accessible_host(host_in, pl->P) &&
+        device_accessible_host(reinterpret_cast<const void *const *>(host_out), pl->P)) {
+      // The kernel reads the inputs from and writes the results to host memory itself.
+      int rc = prepare_fused(pl);
+      if (rc) return rc;
+      return launch_fused_range(pl, host_in, host_out, 0, pl->n, stream);
+    }
+    if (int rc = check_buffers(pl, dev_bufs)) return rc;
+    return run_host_pipelined(pl, host_in, host_out, dev_bufs, stream);
+  }
+  if (int rc = check_buffers(pl, dev_bufs)) return rc;
   for (int x = 0; x < pl->P && bytes; ++x) {
     cudaError_t e = cudaMemcpyAsync(dev_bufs[x], host_in[x], bytes, cudaMemcpyHostToDevice,
                                     (cudaStream_t)stream);

@@ -9,6 +9,7 @@
 #include <algorithm>
 #include <cstdarg>
 #include <cstdio>
+#include <cstdlib>
 #include <functional>
 #include <string>
 #include <vector>
@@ -71,69 +72,69 @@ template <int W> static __device__ __forceinline__ void gar_store(gar_io *p, con
 #if GAR_DTYPE == 1
 template <> __device__ __forceinline__ void gar_load<1>(const gar_io *p, gar_acc *v) {
   gar_u16 h;
-  asm("ld.global.cs.u16 %0, [%1];" : "=h"(h) : "l"(p));
+  asm("ld.global" GAR_LDH ".u16 %0, [%1];" : "=h"(h) : "l"(p));
   v[0] = __uint_as_float(((gar_u32)h) << 16);
 }
 template <> __device__ __forceinline__ void gar_load<2>(const gar_io *p, gar_acc *v) {
   gar_u32 u;
-  asm("ld.global.cs.u32 %0, [%1];" : "=r"(u) : "l"(p));
+  asm("ld.global" GAR_LDH ".u32 %0, [%1];" : "=r"(u) : "l"(p));
   v[0] = gar_bf16_lo(u); v[1] = gar_bf16_hi(u);
 }
 template <> __device__ __forceinline__ void gar_load<4>(const gar_io *p, gar_acc *v) {
   gar_u32 a, b;
-  asm("ld.global.cs.v2.u32 {%0,%1}, [%2];" : "=r"(a), "=r"(b) : "l"(p));
+  asm("ld.global" GAR_LDH ".v2.u32 {%0,%1}, [%2];" : "=r"(a), "=r"(b) : "l"(p));
   v[0] = gar_bf16_lo(a); v[1] = gar_bf16_hi(a); v[2] = gar_bf16_lo(b); v[3] = gar_bf16_hi(b);
 }
 template <> __device__ __forceinline__ void gar_load<8>(const gar_io *p, gar_acc *v) {
   gar_u32 a, b, c, d;
-  asm("ld.global.cs.v4.u32 {%0,%1,%2,%3}, [%4];" : "=r"(a), "=r"(b), "=r"(c), "=r"(d) : "l"(p));
+  asm("ld.global" GAR_LDH ".v4.u32 {%0,%1,%2,%3}, [%4];" : "=r"(a), "=r"(b), "=r"(c), "=r"(d) : "l"(p));
   v[0] = gar_bf16_lo(a); v[1] = gar_bf16_hi(a); v[2] = gar_bf16_lo(b); v[3] = gar_bf16_hi(b);
   v[4] = gar_bf16_lo(c); v[5] = gar_bf16_hi(c); v[6] = gar_bf16_lo(d); v[7] = gar_bf16_hi(d);
 }
 template <> __device__ __forceinline__ void gar_store<1>(gar_io *p, const gar_acc *v) {
   gar_u16 h;
   asm("cvt.rn.bf16.f32 %0, %1;" : "=h"(h) : "f"(v[0]));
-  asm volatile("st.global.cs.u16 [%0], %1;" :: "l"(p), "h"(h) : "memory");
+  asm volatile("st.global" GAR_STH ".u16 [%0], %1;" :: "l"(p), "h"(h) : "memory");
 }
 template <> __device__ __forceinline__ void gar_store<2>(gar_io *p, const gar_acc *v) {
-  asm volatile("st.global.cs.u32 [%0], %1;" :: "l"(p), "r"(gar_pack_bf16(v[0], v[1])) : "memory");
+  asm volatile("st.global" GAR_STH ".u32 [%0], %1;" :: "l"(p), "r"(gar_pack_bf16(v[0], v[1])) : "memory");
 }
 template <> __device__ __forceinline__ void gar_store<4>(gar_io *p, const gar_acc *v) {
-  asm volatile("st.global.cs.v2.u32 [%0], {%1,%2};" :: "l"(p),
+  asm volatile("st.global" GAR_STH ".v2.u32 [%0], {%1,%2};" :: "l"(p),
                "r"(gar_pack_bf16(v[0], v[1])), "r"(gar_pack_bf16(v[2], v[3])) : "memory");
 }
 template <> __device__ __forceinline__ void gar_store<8>(gar_io *p, const gar_acc *v) {
-  asm volatile("st.global.cs.v4.u32 [%0], {%1,%2,%3,%4};" :: "l"(p),
+  asm volatile("st.global" GAR_STH ".v4.u32 [%0], {%1,%2,%3,%4};" :: "l"(p),
                "r"(gar_pack_bf16(v[0], v[1])), "r"(gar_pack_bf16(v[2], v[3])),
                "r"(gar_pack_bf16(v[4], v[5])), "r"(gar_pack_bf16(v[6], v[7])) : "memory");
 }
 #else
 template <> __device__ __forceinline__ void gar_load<1>(const gar_io *p, gar_acc *v) {
   gar_u32 a;
-  asm("ld.global.cs.b32 %0, [%1];" : "=r"(a) : "l"(p));
+  asm("ld.global" GAR_LDH ".b32 %0, [%1];" : "=r"(a) : "l"(p));
   v[0] = *reinterpret_cast<gar_acc *>(&a);
 }
 template <> __device__ __forceinline__ void gar_load<2>(const gar_io *p, gar_acc *v) {
   gar_u32 a, b;
-  asm("ld.global.cs.v2.b32 {%0,%1}, [%2];" : "=r"(a), "=r"(b) : "l"(p));
+  asm("ld.global" GAR_LDH ".v2.b32 {%0,%1}, [%2];" : "=r"(a), "=r"(b) : "l"(p));
   v[0] = *reinterpret_cast<gar_acc *>(&a); v[1] = *reinterpret_cast<gar_acc *>(&b);
 }
 template <> __device__ __forceinline__ void gar_load<4>(const gar_io *p, gar_acc *v) {
   gar_u32 a, b, c, d;
-  asm("ld.global.cs.v4.b32 {%0,%1,%2,%3}, [%4];" : "=r"(a), "=r"(b), "=r"(c), "=r"(d) : "l"(p));
+  asm("ld.global" GAR_LDH ".v4.b32 {%0,%1,%2,%3}, [%4];" : "=r"(a), "=r"(b), "=r"(c), "=r"(d) : "l"(p));
   v[0] = *reinterpret_cast<gar_acc *>(&a); v[1] = *reinterpret_cast<gar_acc *>(&b);
   v[2] = *reinterpret_cast<gar_acc *>(&c); v[3] = *reinterpret_cast<gar_acc *>(&d);
 }
 template <> __device__ __forceinline__ void gar_store<1>(gar_io *p, const gar_acc *v) {
-  asm volatile("st.global.cs.b32 [%0], %1;" :: "l"(p), "r"(*reinterpret_cast<const gar_u32 *>(&v[0])) : "memory");
+  asm volatile("st.global" GAR_STH ".b32 [%0], %1;" :: "l"(p), "r"(*reinterpret_cast<const gar_u32 *>(&v[0])) : "memory");
 }
 template <> __device__ __forceinline__ void gar_store<2>(gar_io *p, const gar_acc *v) {
-  asm volatile("st.global.cs.v2.b32 [%0], {%1,%2};" :: "l"(p),
+  asm volatile("st.global" GAR_STH ".v2.b32 [%0], {%1,%2};" :: "l"(p),
                "r"(*reinterpret_cast<const gar_u32 *>(&v[0])),
                "r"(*reinterpret_cast<const gar_u32 *>(&v[1])) : "memory");
 }
 template <> __device__ __forceinline__ void gar_store<4>(gar_io *p, const gar_acc *v) {
-  asm volatile("st.global.cs.v4.b32 [%0], {%1,%2,%3,%4};" :: "l"(p),
+  asm volatile("st.global" GAR_STH ".v4.b32 [%0], {%1,%2,%3,%4};" :: "l"(p),
                "r"(*reinterpret_cast<const gar_u32 *>(&v[0])),
                "r"(*reinterpret_cast<const gar_u32 *>(&v[1])),
                "r"(*reinterpret_cast<const gar_u32 *>(&v[2])),
@@ -141,6 +142,21 @@ template <> __device__ __forceinline__ void gar_store<4>(gar_io *p, const gar_ac
 }
 #endif
 )CUDA";
+
+// Optional tuning knobs for launch-shape sweeps, read from the environment; each only
+// changes how the same work is laid out (never what is computed), and the chosen values
+// are part of the generated source, so kernels of different settings never share a cache
+// entry.  GAR_TUNE_FUSED_W: elements per thread-vector; GAR_TUNE_FUSED_MINB: minimum
+// resident CTAs per SM in __launch_bounds__; GAR_TUNE_LDH / GAR_TUNE_STH: cache-hint
+// suffix of the global loads / stores (default ".cs", streaming).
+int tune_int(const char *name, int dflt) {
+  const char *v = std::getenv(name);
+  return (v && *v) ? std::atoi(v) : dflt;
+}
+std::string tune_str(const char *name, const char *dflt) {
+  const char *v = std::getenv(name);
+  return (v != nullptr) ? std::string(v) : std::string(dflt);
+}
 
 std::string fmt(const char *f, ...) {
   char buf[1024];
@@ -293,7 +309,11 @@ CodegenResult generate_fused_source(const gar_plan &pl) {
   const FusedProgram &fp = pl.prog;
   const int P = pl.P;
   Schedule sc = order_program(fp);
-  const int W = choose_width(pl.dtype, sc.peak_live, 16);
+  int W = choose_width(pl.dtype, sc.peak_live, 16);
+  if (int w = tune_int("GAR_TUNE_FUSED_W", 0))
+    if (w > 0 && (w & (w - 1)) == 0 && w * elem_size(pl.dtype) <= 16) W = w;
+  const int minb = tune_int("GAR_TUNE_FUSED_MINB", 0);
+  const std::string bounds = minb > 0 ? fmt("__launch_bounds__(256, %d)", minb) : "__launch_bounds__(256)";
   const bool rotate = pl.K != P;   // latency-optimal results do not depend on the block
   CodegenResult cg;
   cg.width = W;
@@ -301,19 +321,25 @@ CodegenResult generate_fused_source(const gar_plan &pl) {
                    op_tag(pl.op) + fmt("_W%d", W);
   std::string s;
   s += fmt("#define GAR_DTYPE %d\n#define GAR_OP %d\n", pl.dtype, pl.op);
+  s += "#define GAR_LDH \"" + tune_str("GAR_TUNE_LDH", ".cs") + "\"\n";
+  s += "#define GAR_STH \"" + tune_str("GAR_TUNE_STH", ".cs") + "\"\n";
   s += kSkeleton;
   s += fmt("#define GAR_P %d\n#define GAR_W %d\n", P, W);
   s += fmt("#define GAR_N %lluULL\n", (unsigned long long)pl.n);
-  s += fmt("struct gar_args { gar_io *rank[%d]; };\n", P);
+  // in[] / out[]: where rank x's contributions are read and its results written (equal
+  // for the in-place Allreduce); [e_lo, e_hi): the element positions this launch covers
+  // (e_lo a multiple of GAR_W), so one Allreduce can run as several launches.
+  s += fmt("struct gar_args { const gar_io *in[%d]; gar_io *out[%d]; gar_u64 e_lo, e_hi; };\n", P, P);
   s += emit_block_of("gar_block_of", P, pl.n);
-  auto row = [](const std::string &r) { return "a.rank[" + r + "]"; };
-  s += emit_eval(fp, sc, "plan", "const gar_args &a", row, row, rotate);
-  s += "extern \"C\" __global__ void __launch_bounds__(256) " + cg.kernel_name +
+  auto ld_row = [](const std::string &r) { return "a.in[" + r + "]"; };
+  auto st_row = [](const std::string &r) { return "a.out[" + r + "]"; };
+  s += emit_eval(fp, sc, "plan", "const gar_args &a", ld_row, st_row, rotate);
+  s += "extern \"C\" __global__ void " + bounds + " " + cg.kernel_name +
        "(const __grid_constant__ gar_args a) {\n";
-  s += "  const gar_u64 nvec = GAR_N / GAR_W;\n";
+  s += "  const gar_u64 v_lo = a.e_lo / GAR_W, v_hi = a.e_hi / GAR_W;\n";
   s += "  const gar_u64 stride = (gar_u64)gridDim.x * blockDim.x;\n";
   s += "  const gar_u64 tid = (gar_u64)blockIdx.x * blockDim.x + threadIdx.x;\n";
-  s += "  for (gar_u64 v = tid; v < nvec; v += stride) {\n";
+  s += "  for (gar_u64 v = v_lo + tid; v < v_hi; v += stride) {\n";
   s += "    const gar_u64 e0 = v * GAR_W;\n";
   if (rotate) {
     s += "    const int b0 = gar_block_of(e0);\n";
@@ -326,9 +352,9 @@ CodegenResult generate_fused_source(const gar_plan &pl) {
     s += "    gar_eval_plan<GAR_W>(a, e0, 0);\n";
   }
   s += "  }\n";
-  s += "  const gar_u64 tail = GAR_N - nvec * GAR_W;\n";
-  s += "  if (tid < tail) {\n";
-  s += "    const gar_u64 e = nvec * GAR_W + tid;\n";
+  s += "  const gar_u64 t0 = (v_hi * GAR_W > a.e_lo ? v_hi * GAR_W : a.e_lo);\n";
+  s += "  if (tid < a.e_hi - t0) {\n";
+  s += "    const gar_u64 e = t0 + tid;\n";
   s += rotate ? "    gar_eval_plan<1>(a, e, gar_block_of(e));\n" : "    gar_eval_plan<1>(a, e, 0);\n";
   s += "  }\n}\n";
   cg.source = s;
@@ -353,6 +379,8 @@ CodegenResult generate_batched_source(const std::vector<const gar_plan *> &plans
   cg.kernel_name = name + dtype_tag(p0.dtype) + "_" + op_tag(p0.op) + fmt("_W%d", W);
   std::string s;
   s += fmt("#define GAR_DTYPE %d\n#define GAR_OP %d\n", p0.dtype, p0.op);
+  s += "#define GAR_LDH \"" + tune_str("GAR_TUNE_LDH", ".cs") + "\"\n";
+  s += "#define GAR_STH \"" + tune_str("GAR_TUNE_STH", ".cs") + "\"\n";
   s += kSkeleton;
   s += fmt("#define GAR_W %d\n#define GAR_N %lluULL\n", W, (unsigned long long)p0.n);
   s += "struct gar_desc { int plan; int reserved; const void *in; void *out; };\n";

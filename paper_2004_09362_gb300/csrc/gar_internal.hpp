@@ -63,6 +63,8 @@ struct FusedProgram {
 
 struct JitKernel;  // jit.cpp
 
+constexpr int GAR_HOST_CHUNKS_MAX = 16;  // element chunks of the pipelined host path
+
 }  // namespace gar
 
 struct gar_plan {
@@ -89,6 +91,12 @@ struct gar_plan {
   bool ran_step_faithful = false;
   gar::JitKernel *fused = nullptr;   // owned by the JIT cache
   int fused_width = 0;
+  // pipelined host-buffer path: 3 streams (to device, kernel, to host) and events
+  bool hp_ready = false;
+  void *hp_stream[3] = {nullptr, nullptr, nullptr};
+  void *hp_h2d[gar::GAR_HOST_CHUNKS_MAX] = {};
+  void *hp_krn[gar::GAR_HOST_CHUNKS_MAX] = {};
+  void *hp_start = nullptr, *hp_done = nullptr;
 };
 
 namespace gar {

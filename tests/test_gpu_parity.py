@@ -333,20 +333,31 @@ def test_batched_mixed_order_and_steps():
 # Host-buffer entry point and argument handling on the device
 # ---------------------------------------------------------------------------
 
+@pytest.mark.parametrize("layout", ["pinned", "pinned_misaligned", "pageable"])
+@pytest.mark.parametrize("P,n,dtype,S", [(7, 70001, "f32", 4), (5, 16 * 65536 + 37, "bf16", 5),
+                                         (24, 3 * 65536 + 5, "f32", 10), (6, 1000, "i32", 3)])
 @pytest.mark.parametrize("mode", ["fused", "step"])
-def test_host_buffers(mode):
-    P, n = 7, 70001
-    t = _np_inputs(P, n, "f32", seed=11)
-    host_in = t.clone().pin_memory()
-    host_out = torch.empty_like(host_in).pin_memory()
+def test_host_buffers(P, n, dtype, S, mode, layout):
+    """gar_allreduce_host.  Fused mode on aligned host memory the GPU can address runs
+    the kernel on the host buffers directly; misaligned host rows take the staged path
+    (copies in element chunks pipelined over internal streams, several chunks and a
+    ragged last chunk here); step-faithful mode copies, reduces, copies back."""
+    t = _np_inputs(P, n, dtype, seed=11)
+    off = 1 if layout == "pinned_misaligned" else 0
+    host_in = torch.zeros((P, n + off), dtype=t.dtype)
+    host_in[:, off:] = t
+    host_out = torch.zeros_like(host_in)
+    if layout != "pageable":
+        host_in, host_out = host_in.pin_memory(), host_out.pin_memory()
     dev_store, _ = _padded_device(t)
-    plan = gar.gar_plan_create(P, n, "f32", "sum", 4)
-    rows_in = [host_in[x] for x in range(P)]
-    rows_out = [host_out[x] for x in range(P)]
+    plan = gar.gar_plan_create(P, n, dtype, "sum", S)
+    rows_in = [host_in[x, off:] for x in range(P)]
+    rows_out = [host_out[x, off:] for x in range(P)]
     gar.gar_allreduce_host(plan, rows_in, rows_out, dev_store, mode)
     torch.cuda.synchronize()
-    want = G.allreduce(_to_host_list(t, "f32"), 4, "sum", "f32")
-    _assert_same(host_out, want, "f32", "host")
+    want = G.allreduce(_to_host_list(t, dtype), S, "sum", dtype)
+    _assert_same(host_out[:, off:], want, dtype, "host")
+    assert bool((host_in[:, off:] == t).all())        # inputs untouched
 
 
 def test_missing_workspace_is_an_error():
