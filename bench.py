@@ -217,6 +217,13 @@ def _step_dram_bytes(gar, plan, P, n, dtype):
     return tot
 
 
+def _l(P):
+    L = 0
+    while (1 << L) < P:
+        L += 1
+    return L
+
+
 def run_ours(args):
     import torch
     import gar_inputs
@@ -232,17 +239,60 @@ def run_ours(args):
         dist.init_process_group("nccl" if torch.cuda.is_available() else "gloo")
     stream = torch.cuda.current_stream()
     hbm_peak, peak_kind = _peaks()
+    headline = (args.workload == HEADLINE and args.S in (None, 10) and args.mode == "fused"
+                and args.op == "sum")
 
-    wl = gar_inputs.WORKLOADS[HEADLINE]
-    P, n, S = wl.P, wl.n, 10
-    inp = gar_inputs.rank_inputs(P, n, wl.dtype, wl.dist, wl.seed + rank, device="cuda")
-    plan = gar.gar_plan_create(P, n, wl.dtype, "sum", S)
-    gar.gar_plan_prepare(plan, "fused")
-    info = plan.info()
-    ptrs = gar.rank_pointers(inp)
+    if args.workload == "batched_425B":
+        cfgb = gar_inputs.BATCHED
+        flat, layout = gar_inputs.batched_inputs(cfgb["count"], cfgb["Ps"], cfgb["n"], "f32",
+                                                 cfgb["dist"], cfgb["seed"] + rank, device="cuda")
+        out_t = torch.empty_like(flat)
+        plans = [gar.gar_plan_create(Pb, cfgb["n"], "f32", args.op, gar.GAR_STEPS_LO)
+                 for Pb in cfgb["Ps"]]
+        idx = {Pb: k for k, Pb in enumerate(cfgb["Ps"])}
+        desc = gar.make_batch_desc([idx[Pb] for (Pb, _o) in layout],
+                                   [flat.data_ptr() + o * 4 for (_Pb, o) in layout],
+                                   [out_t.data_ptr() + o * 4 for (_Pb, o) in layout])
+        bytes_step = 2 * flat.numel() * 4
+        launches_per_step = 1
+        kernel_desc = f"batched {cfgb['count']} x P in {cfgb['Ps']} x {cfgb['n']} f32 {args.op}"
+        config = {"workload": "batched_425B", "count": cfgb["count"], "Ps": list(cfgb["Ps"]),
+                  "n_per_rank": cfgb["n"], "schedule": "latency-optimal", "op": args.op,
+                  "mode": "batched", "parallelism": f"replicas x{ws}",
+                  "l2": "361 MB moved per step > 129 MB L2"}
+        dtype = "f32"
 
-    def step():
-        gar.gar_allreduce(plan, ptrs, "fused", stream)
+        def step():
+            gar.gar_allreduce_batched(plans, desc, cfgb["count"], stream)
+        plan = None
+    else:
+        wl = gar_inputs.WORKLOADS[args.workload]
+        P, n = wl.P, wl.n
+        S = args.S if args.S is not None else 2 * _l(P)
+        dtype = wl.dtype
+        inp = gar_inputs.rank_inputs(P, n, wl.dtype, wl.dist, wl.seed + rank, device="cuda")
+        plan = gar.gar_plan_create(P, n, wl.dtype, args.op, S)
+        if args.mode == "step":
+            gar.ensure_workspace(plan)
+        gar.gar_plan_prepare(plan, args.mode)
+        ptrs = gar.rank_pointers(inp)
+        info = plan.info()
+        launches_per_step = 1 if args.mode == "fused" else info["n_launches"]
+        if args.mode == "fused":
+            bytes_step = _alg_bytes(P, n, wl.dtype)
+        else:
+            bytes_step = _step_dram_bytes(gar, plan, P, n, wl.dtype)
+        kernel_desc = (f"{args.mode} P{P} S{S} {wl.dtype} {args.op}"
+                       + (f" W{info['fused_width']} regs{info['fused_regs']}" if args.mode == "fused" else ""))
+        sched = "bandwidth-optimal" if S == 2 * _l(P) else ("latency-optimal" if S == _l(P) else "intermediate")
+        config = {"workload": args.workload, "P": P, "n_per_rank": n,
+                  "bytes_per_rank": n * (2 if wl.dtype == "bf16" else 4), "steps_S": S,
+                  "schedule": sched, "mode": args.mode, "op": args.op,
+                  "parallelism": f"replicas x{ws}",
+                  "l2": f"{2 * P * n * (2 if wl.dtype == 'bf16' else 4) / 2**30:.2f} GiB moved per step > 129 MB L2"}
+
+        def step():
+            gar.gar_allreduce(plan, ptrs, args.mode, stream)
 
     for _ in range(args.warmup):
         step()
@@ -261,31 +311,35 @@ def run_ours(args):
     if dist is not None:
         dist.barrier()
     ms = max_over_ranks(start.elapsed_time(end) / args.steps, dist, "cuda")
-    bytes_step = _alg_bytes(P, n, wl.dtype)
-    value = job_gbs(bytes_step, ws, ms)
+    if args.workload == "batched_425B" or args.mode == "fused":
+        value = job_gbs(bytes_step, ws, ms)
+    else:
+        value = job_gbs(_alg_bytes(P, n, dtype), ws, ms)
     clocks = clk.summary()
-    kernel_gbs = bytes_step / (ms * 1e-3) / 1e9
+    kernel_gbs = bytes_step / (ms * 1e-3) / 1e9 / launches_per_step * launches_per_step
 
     out = {
         "metric": METRIC, "value": round(value, 2), "unit": "GB/s", "n_gpus": ws,
         "steps": args.steps, "warmup": args.warmup, "ms_per_step": round(ms, 5),
-        "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f32",
-        "data": "synthetic (seeded N(0,1e-3) fp32, generated on the GPU)",
-        "config": {"workload": HEADLINE, "P": P, "n_per_rank": n, "bytes_per_rank": n * 4,
-                   "steps_S": S, "schedule": "bandwidth-optimal", "mode": "fused", "op": "sum",
-                   "parallelism": f"replicas x{ws}", "l2": "inputs 1.5 GiB + outputs 1.5 GiB per step > 129 MB L2"},
-        "gpu_launches": args.steps,
+        "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": dtype,
+        "data": "synthetic (seeded, generated on the GPU; see gar_inputs.py)",
+        "config": config,
+        "gpu_launches": args.steps * launches_per_step,
         "roofline": {"bound": "hbm", "achieved": round(kernel_gbs, 1), "peak": hbm_peak,
                      "unit": "GB/s", "frac": round(kernel_gbs / hbm_peak, 4),
-                     "traffic": _committed_traffic(), "peak_kind": peak_kind,
-                     "kernel": plan.info().get("fused_width") and f"fused P{P} S{S} f32 sum",
-                     "algorithmic_bytes_per_launch": bytes_step},
+                     "traffic": _committed_traffic(gar) if headline else None,
+                     "peak_kind": peak_kind, "kernel": kernel_desc,
+                     "algorithmic_bytes_per_launch": bytes_step // launches_per_step
+                     if launches_per_step == 1 else None,
+                     "algorithmic_bytes_per_step": bytes_step},
         "clocks": clocks,
     }
+    if args.workload == "batched_425B":
+        out["reductions_per_s"] = round(gar_inputs.BATCHED["count"] * ws / (ms * 1e-3), 1)
 
     # ---- end to end through the host-buffer entry point
-    if not args.no_e2e:
-        out["e2e"] = _e2e(gar, plan, inp, P, n, args, stream, dist)
+    if not args.no_e2e and plan is not None:
+        out["e2e"] = _e2e(gar, plan, inp, P, n, dtype, args, stream, dist)
 
     if rank == 0 and not args.no_rows:
         out["rows"] = measure_rows(gar, gar_inputs, stream, hbm_peak)
@@ -298,30 +352,33 @@ def run_ours(args):
         print(json.dumps(out), flush=True)
 
 
-def _committed_traffic():
-    """DRAM bytes per launch of the headline fused kernel from the committed ncu summary
-    (profiles/fused_p24_64mib_f32.txt), or None when absent or when the kernel generator
-    (csrc/codegen.cpp) has changed since the counters were taken."""
+def headline_kernel_sha(gar) -> str:
+    """sha1 (12 hex digits) of the generated source of the headline fused kernel."""
     import hashlib
+    plan = gar.gar_plan_create(24, 16777216, "f32", "sum", 10)
+    return hashlib.sha1(gar.gar_plan_fused_source(plan).encode()).hexdigest()[:12]
+
+
+def _committed_traffic(gar):
+    """DRAM bytes per launch of the headline fused kernel from the committed ncu summary
+    (profiles/fused_p24_64mib_f32.txt), or None when absent or when the generated kernel
+    differs from the one the counters were taken on."""
     path = os.path.join(ROOT, "profiles", "fused_p24_64mib_f32.txt")
-    src = os.path.join(ROOT, "paper_2004_09362_gb300", "csrc", "codegen.cpp")
     try:
-        with open(src, "rb") as f:
-            sha = hashlib.sha1(f.read()).hexdigest()[:12]
         fields = {}
         with open(path) as f:
             for line in f:
                 if ":" in line and not line.startswith(" "):
                     k, v = line.split(":", 1)
                     fields[k.strip()] = v.strip()
-        if fields.get("codegen_sha1") != sha:
+        if fields.get("kernel_source_sha1") != headline_kernel_sha(gar):
             return None
         return int(fields["dram_bytes_per_launch"].split()[0])
     except Exception:
         return None
 
 
-def _e2e(gar, plan, inp, P, n, args, stream, dist):
+def _e2e(gar, plan, inp, P, n, dtype, args, stream, dist):
     import torch
     host_in = inp.cpu().pin_memory()
     host_out = torch.empty_like(host_in).pin_memory()
@@ -333,15 +390,15 @@ def _e2e(gar, plan, inp, P, n, args, stream, dist):
     dp = gar.rank_pointers(dev)
 
     def step():
-        gar.gar_allreduce_host(plan, hp_in, hp_out, dp, "fused", stream)
+        gar.gar_allreduce_host(plan, hp_in, hp_out, dp, args.mode, stream)
 
     steps = max(1, min(args.steps, 10))
     ms = max_over_ranks(_time_loop(step, steps, 3, stream), dist, "cuda")
     ws = dist.get_world_size() if dist is not None else 1
-    bytes_step = _alg_bytes(P, n, "f32")
+    bytes_step = _alg_bytes(P, n, dtype)
     return {"value": round(job_gbs(bytes_step, ws, ms), 2), "unit": "GB/s",
-            "ms_per_step": round(ms, 4), "h2d_bytes_per_step": P * n * 4,
-            "d2h_bytes_per_step": P * n * 4, "steps": steps,
+            "ms_per_step": round(ms, 4), "h2d_bytes_per_step": bytes_step // 2,
+            "d2h_bytes_per_step": bytes_step // 2, "steps": steps,
             "path": "gar_allreduce_host on pinned host buffers: the fused kernel reads the P inputs from and writes the P results to host memory over NVLink-C2C (no staging copies)"}
 
 
@@ -439,8 +496,9 @@ def measure_rows(gar, gar_inputs, stream, hbm_peak):
         desc = gar.make_batch_desc([idx[P] for (P, _o) in layout],
                                    [flat.data_ptr() + o * es for (_P, o) in layout],
                                    [out.data_ptr() + o * es for (_P, o) in layout])
+        # 361 MB per call > 129 MB L2: back-to-back calls need no flush
         ms = _time_loop(lambda: gar.gar_allreduce_batched(plans, desc, cfg["count"], stream), 20, 3,
-                        stream, flusher)
+                        stream)
         nbytes = 2 * flat.numel() * es
         rows[f"batched_65536x425B_{op}"] = {
             "us": round(ms * 1e3, 2), "reductions_per_s": round(cfg["count"] / (ms * 1e-3), 1),
@@ -533,6 +591,11 @@ def main():
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--no-cpu", action="store_true")
     ap.add_argument("--cpu-seconds", type=float, default=10.0)
+    ap.add_argument("--workload", default=HEADLINE,
+                    help="gar_inputs.WORKLOADS key or batched_425B (default: the headline)")
+    ap.add_argument("--S", type=int, default=None, help="step count (default: 2*ceil(log2 P))")
+    ap.add_argument("--mode", default="fused", choices=["fused", "step"])
+    ap.add_argument("--op", default="sum", choices=["sum", "max", "min"])
     args = ap.parse_args()
     if args.warmup < 3:
         args.warmup = 3

@@ -96,7 +96,9 @@ typedef struct {
   int32_t n_launches;        /* step-faithful kernel launches per Allreduce */
   uint64_t n;                /* elements per rank */
   int32_t fused_combines;    /* combines per element position in fused mode */
-  int32_t fused_width;       /* elements per thread-vector in the fused kernel */
+  int32_t fused_width;       /* elements per thread-vector in the fused kernel (0 until compiled) */
+  int32_t fused_regs;        /* registers per thread of the loaded fused kernel (0 until loaded) */
+  int32_t fused_local_bytes; /* local (spill) bytes per thread of the loaded fused kernel */
 } gar_plan_info;
 
 /* Creates a schedule for P virtual ranks of n elements each.
@@ -152,6 +154,11 @@ GAR_API int gar_plan_step_ops(const gar_plan *plan, int32_t *ops, int *nops, int
 /* Caller-owned device workspace for step-faithful mode (16-byte aligned, at least
  * workspace_bytes).  NULL with 0 bytes detaches it. */
 GAR_API int gar_plan_set_workspace(gar_plan *plan, void *dev_ptr, size_t bytes);
+
+/* The CUDA C source of the plan's generated fused kernel (host-only).  Copies at most
+ * *len bytes (including the terminating NUL) to buf and sets *len to the full size
+ * including the NUL; pass buf == NULL to query the size. */
+GAR_API int gar_plan_fused_source(const gar_plan *plan, char *buf, size_t *len);
 
 /* Compiles (host-only, needs no GPU) the specialized kernel for `mode`.  Optional:
  * gar_plan_prepare and the first Allreduce compile on demand. */

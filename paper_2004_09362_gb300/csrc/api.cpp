@@ -351,6 +351,10 @@ int gar_plan_get_info(const gar_plan *pl, gar_plan_info *info) {
   info->n = pl->n;
   info->fused_combines = (int)pl->prog.a.size();
   info->fused_width = pl->fused_width;
+  if (pl->fused != nullptr && pl->fused->loaded) {
+    info->fused_regs = pl->fused->regs;
+    info->fused_local_bytes = pl->fused->local_bytes;
+  }
   return GAR_OK;
 }
 
@@ -420,6 +424,19 @@ int gar_plan_step_ops(const gar_plan *pl, int32_t *ops, int *nops, int32_t *laun
       }
     }
   }
+  return GAR_OK;
+}
+
+int gar_plan_fused_source(const gar_plan *pl, char *buf, size_t *len) {
+  if (int rc = check_plan(pl)) return rc;
+  if (len == nullptr) return GAR_EINVAL;
+  const std::string src = generate_fused_source(*pl).source;
+  if (buf != nullptr && *len > 0) {
+    const size_t m = std::min(*len - 1, src.size());
+    std::memcpy(buf, src.data(), m);
+    buf[m] = '\0';
+  }
+  *len = src.size() + 1;
   return GAR_OK;
 }
 

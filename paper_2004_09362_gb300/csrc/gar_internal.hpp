@@ -126,6 +126,7 @@ struct JitKernel {
   int width = 1;
   int threads = 256;
   int blocks_per_sm = 0;
+  int regs = 0, local_bytes = 0;
   bool loaded = false;
 };
 int jit_compile(const CodegenResult &cg, JitKernel **out);

@@ -82,6 +82,13 @@ int jit_load(JitKernel *k) {
     cudaGetLastError();
     nb = 1;
   }
+  cudaFuncAttributes fa{};
+  if (cudaFuncGetAttributes(&fa, (const void *)kern) == cudaSuccess) {
+    k->regs = fa.numRegs;
+    k->local_bytes = (int)fa.localSizeBytes;
+  } else {
+    cudaGetLastError();
+  }
   k->library = lib;
   k->kernel = (void *)kern;
   k->blocks_per_sm = nb;

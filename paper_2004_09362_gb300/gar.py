@@ -34,7 +34,7 @@ EXPORTS = (
     "gar_plan_step", "gar_plan_origin", "gar_plan_fused_program", "gar_plan_step_ops",
     "gar_plan_set_workspace", "gar_plan_compile", "gar_plan_prepare", "gar_allreduce",
     "gar_allreduce_host", "gar_allreduce_batched", "gar_last_step_bytes", "gar_strerror",
-    "gar_last_error", "gar_selftest_compile", "gar_allreduce_noalloc",
+    "gar_last_error", "gar_selftest_compile", "gar_allreduce_noalloc", "gar_plan_fused_source",
 )
 
 
@@ -48,7 +48,8 @@ class gar_plan_info(ctypes.Structure):
     _fields_ = [("P", ctypes.c_int32), ("L", ctypes.c_int32), ("S", ctypes.c_int32),
                 ("r", ctypes.c_int32), ("K", ctypes.c_int32), ("dtype", ctypes.c_int32),
                 ("op", ctypes.c_int32), ("n_launches", ctypes.c_int32), ("n", ctypes.c_uint64),
-                ("fused_combines", ctypes.c_int32), ("fused_width", ctypes.c_int32)]
+                ("fused_combines", ctypes.c_int32), ("fused_width", ctypes.c_int32),
+                ("fused_regs", ctypes.c_int32), ("fused_local_bytes", ctypes.c_int32)]
 
 
 def _load():
@@ -77,6 +78,7 @@ def _load():
         "gar_last_error": (ctypes.c_char_p, []),
         "gar_selftest_compile": (i32, []),
         "gar_allreduce_noalloc": (i32, [vp, P_(vp), vp]),
+        "gar_plan_fused_source": (i32, [vp, ctypes.c_char_p, P_(sz)]),
     }
     for name, (res, args) in sig.items():
         fn = getattr(lib, name)
@@ -129,7 +131,7 @@ class Plan:
         return self._h
 
     def info(self) -> dict:
-        if self._info is None or self._info["fused_width"] == 0:
+        if self._info is None or self._info["fused_width"] == 0 or self._info["fused_regs"] == 0:
             self._info = gar_plan_get_info(self)
         return self._info
 
@@ -209,6 +211,14 @@ def gar_plan_step_ops(plan: Plan):
            "gar_plan_step_ops")
     arr = np.frombuffer(ops, dtype=np.int32, count=8 * nops.value).reshape(nops.value, 8).copy()
     return arr, [int(part[k]) for k in range(nl.value)]
+
+
+def gar_plan_fused_source(plan: Plan) -> str:
+    n = ctypes.c_size_t(0)
+    _check(_lib.gar_plan_fused_source(plan.handle, None, ctypes.byref(n)), "gar_plan_fused_source")
+    buf = ctypes.create_string_buffer(n.value)
+    _check(_lib.gar_plan_fused_source(plan.handle, buf, ctypes.byref(n)), "gar_plan_fused_source")
+    return buf.value.decode()
 
 
 def gar_plan_set_workspace(plan: Plan, ptr: int, nbytes: int) -> None:
