@@ -399,7 +399,11 @@ def _e2e(gar, plan, inp, P, n, dtype, args, stream, dist):
     return {"value": round(job_gbs(bytes_step, ws, ms), 2), "unit": "GB/s",
             "ms_per_step": round(ms, 4), "h2d_bytes_per_step": bytes_step // 2,
             "d2h_bytes_per_step": bytes_step // 2, "steps": steps,
-            "path": "gar_allreduce_host on pinned host buffers: the fused kernel reads the P inputs from and writes the P results to host memory over NVLink-C2C (no staging copies)"}
+            "path": ("gar_allreduce_host on pinned host buffers: the fused kernel reads the P inputs "
+                     "from and writes the P results to host memory over NVLink-C2C (no staging copies)")
+            if args.mode == "fused" else
+            ("gar_allreduce_host: P cudaMemcpyAsync to device buffers, the step-faithful "
+             "launches, P cudaMemcpyAsync back, on one stream")}
 
 
 def measure_rows(gar, gar_inputs, stream, hbm_peak):

@@ -20,8 +20,19 @@
 namespace gar {
 namespace {
 
+#ifndef GAR_STEP_CHUNK
+#define GAR_STEP_CHUNK 16384
+#endif
+#ifndef GAR_STEP_UNROLL
+#define GAR_STEP_UNROLL 2
+#endif
+// Launch shape, from a sweep on GB300 (P=24 x 64 MiB fp32, P=127 x 8 MiB bf16, P=8 x
+// 1 MiB): CTAs own 16384-element chunks (smaller chunks ran up to 2.5x slower) and each
+// thread issues the loads of 2 vectors before combining.  Small vectors drop the chunk
+// to 8192 or 4096 elements to keep at least 4 CTAs per SM.
 constexpr int kThreads = 256;
-constexpr uint64_t kChunk = 8192;  // elements per CTA
+constexpr uint64_t kChunk = GAR_STEP_CHUNK;  // largest chunk (elements per CTA)
+constexpr int kUnroll = GAR_STEP_UNROLL;     // 4-element vectors a thread loads at once
 
 template <int MAXP>
 struct StepArgs {
@@ -30,6 +41,7 @@ struct StepArgs {
   const StepOp *ops;                 // this launch's ops
   unsigned long long *bytes;         // counter of the communication step, or nullptr
   uint64_t q, rem, n_pad;
+  uint64_t chunk;                    // elements per CTA
   int P, partner, nops, nchunks;
 };
 
@@ -130,10 +142,10 @@ __global__ void __launch_bounds__(kThreads) step_kernel(const __grid_constant__ 
   const int b = ((x - (int)op.dst_place) % a.P + a.P) % a.P;
   const uint64_t bstart = (uint64_t)b * a.q + ((uint64_t)b < a.rem ? (uint64_t)b : a.rem);
   const uint64_t blen = a.q + ((uint64_t)b < a.rem ? 1 : 0);
-  const uint64_t c0 = (uint64_t)chunk * kChunk;
+  const uint64_t c0 = (uint64_t)chunk * a.chunk;
   if (c0 >= blen) return;
   const uint64_t lo = bstart + c0;
-  const uint64_t hi = bstart + (blen < c0 + kChunk ? blen : c0 + kChunk);
+  const uint64_t hi = bstart + (blen < c0 + a.chunk ? blen : c0 + a.chunk);
 
   const bool has_recv = op.recv_place >= 0;
   const int partner = ((x + a.partner) % a.P + a.P) % a.P;
@@ -156,35 +168,38 @@ __global__ void __launch_bounds__(kThreads) step_kernel(const __grid_constant__ 
     store1<T, A>(op.out0_buf, out0, e, o0);
     if (out1) store1<T, A>(op.out1_buf, out1, e, o1);
   };
-  auto do4 = [&](uint64_t e) {
-    A r[4] = {A(0), A(0), A(0), A(0)};
-    if (has_recv) {
-      load4<T, A>(op.recv_buf, recv, e, r);
-      moved += 4;
-    }
-    A o0[4], o1[4];
-    if (own0) {
-      load4<T, A>(op.out0_own, own0, e, o0);
-      if (has_recv)
+  // kUnroll aligned 4-element vectors per thread: every load of the batch is issued
+  // before the first combine, so a thread keeps up to 3 * kUnroll 16-byte loads in flight.
+  auto do4xU = [&](uint64_t e_first, uint64_t stride, uint64_t vend) {
+    A r[kUnroll][4], o0[kUnroll][4], o1[kUnroll][4];
 #pragma unroll
-        for (int k = 0; k < 4; ++k) o0[k] = combine<OP>(o0[k], r[k]);
-    } else {
-#pragma unroll
-      for (int k = 0; k < 4; ++k) o0[k] = r[k];
-    }
-    if (out1) {
-      if (own1) {
-        load4<T, A>(op.out1_own, own1, e, o1);
-        if (has_recv)
-#pragma unroll
-          for (int k = 0; k < 4; ++k) o1[k] = combine<OP>(o1[k], r[k]);
-      } else {
-#pragma unroll
-        for (int k = 0; k < 4; ++k) o1[k] = r[k];
+    for (int u = 0; u < kUnroll; ++u) {
+      const uint64_t e = e_first + u * stride;
+      if (e < vend) {
+        if (has_recv) {
+          load4<T, A>(op.recv_buf, recv, e, r[u]);
+          moved += 4;
+        }
+        if (own0) load4<T, A>(op.out0_own, own0, e, o0[u]);
+        if (out1 && own1) load4<T, A>(op.out1_own, own1, e, o1[u]);
       }
     }
-    store4<T, A>(op.out0_buf, out0, e, o0);
-    if (out1) store4<T, A>(op.out1_buf, out1, e, o1);
+#pragma unroll
+    for (int u = 0; u < kUnroll; ++u) {
+      const uint64_t e = e_first + u * stride;
+      if (e < vend) {
+#pragma unroll
+        for (int k = 0; k < 4; ++k) {
+          if (!has_recv) {
+            r[u][k] = A(0);
+          }
+          o0[u][k] = own0 ? (has_recv ? combine<OP>(o0[u][k], r[u][k]) : o0[u][k]) : r[u][k];
+          if (out1) o1[u][k] = own1 ? (has_recv ? combine<OP>(o1[u][k], r[u][k]) : o1[u][k]) : r[u][k];
+        }
+        store4<T, A>(op.out0_buf, out0, e, o0[u]);
+        if (out1) store4<T, A>(op.out1_buf, out1, e, o1[u]);
+      }
+    }
   };
 
   // Element offsets are the same in every buffer, and every buffer base is 16-byte
@@ -194,7 +209,8 @@ __global__ void __launch_bounds__(kThreads) step_kernel(const __grid_constant__ 
   if (va > hi) va = hi;
   if (vb < va) vb = va;
   for (uint64_t e = lo + threadIdx.x; e < va; e += blockDim.x) do1(e);
-  for (uint64_t e = va + 4 * (uint64_t)threadIdx.x; e < vb; e += 4 * (uint64_t)blockDim.x) do4(e);
+  const uint64_t vstride = 4 * (uint64_t)blockDim.x;
+  for (uint64_t e = va + 4 * (uint64_t)threadIdx.x; e < vb; e += kUnroll * vstride) do4xU(e, vstride, vb);
   for (uint64_t e = vb + threadIdx.x; e < hi; e += blockDim.x) do1(e);
 
   if (a.bytes != nullptr && has_recv) {
@@ -204,6 +220,20 @@ __global__ void __launch_bounds__(kThreads) step_kernel(const __grid_constant__ 
     const unsigned long long esize = (op.recv_buf == BUF_RANK) ? sizeof(T) : sizeof(A);
     if ((threadIdx.x & 31) == 0 && m) atomicAdd(a.bytes, m * esize);
   }
+}
+
+int num_sms() {
+  static int sms = 0;
+  if (sms == 0) {
+    int dev = 0, v = 0;
+    cudaGetDevice(&dev);
+    if (cudaDeviceGetAttribute(&v, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess || v <= 0) {
+      cudaGetLastError();
+      v = 1;
+    }
+    sms = v;
+  }
+  return sms;
 }
 
 template <typename T, int OP, int MAXP>
@@ -230,7 +260,10 @@ int launch_typed(const gar_plan &pl, const Launch &ln, int launch_index, void *c
   a.partner = ln.partner;
   a.nops = ln.nops;
   const uint64_t maxblk = pl.q + (pl.rem ? 1 : 0);
-  a.nchunks = (int)((maxblk + kChunk - 1) / kChunk);
+  a.chunk = kChunk;
+  const uint64_t min_ctas = 4 * (uint64_t)num_sms();
+  while (a.chunk > 4096 && ((maxblk + a.chunk - 1) / a.chunk) * pl.P * ln.nops < min_ctas) a.chunk /= 2;
+  a.nchunks = (int)((maxblk + a.chunk - 1) / a.chunk);
   if (a.nchunks == 0 || ln.nops == 0) return GAR_OK;
   const uint64_t grid = (uint64_t)a.nchunks * (uint64_t)pl.P * (uint64_t)ln.nops;
   if (grid > 0x7fffffffull) {
