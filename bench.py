@@ -507,7 +507,78 @@ def measure_rows(gar, gar_inputs, stream, hbm_peak):
         rows[f"batched_65536x425B_{op}"] = {
             "us": round(ms * 1e3, 2), "reductions_per_s": round(cfg["count"] / (ms * 1e-3), 1),
             "GB/s": round(nbytes / ms / 1e6, 1), "frac": round(nbytes / ms / 1e6 / hbm_peak, 4)}
+    del flat, out
+    torch.cuda.empty_cache()
+    rows["cost_model_p127_bf16_step"] = cost_model_row(gar, gar_inputs, stream)
     return rows
+
+
+def _paper_blocks(P, S):
+    """Per-rank traffic and combine counts in blocks of the paper's cost model (eqs.
+    bo_cost, intemediate_cost, lo_cost)."""
+    L = _l(P)
+    r = 2 * L - S
+    if r == L:
+        return P * L, P * (2 * L - 2)
+    extra = 2 ** r - 1
+    return 2 * (P - 1) + extra * (L - 1), (P - 1) + extra * (2 * L - 2)
+
+
+def cost_model_row(gar, gar_inputs, stream, P=127, dtype="bf16",
+                   sizes=(425, 9 * 1024, 64 * 1024, 512 * 1024, 4 << 20, 8 << 20)):
+    """Step-faithful mode as the paper's machine: measure every step count at several
+    message sizes, fit the cost model's alpha (per step), beta (per byte moved) and gamma
+    (per byte combined) by non-negative least squares on relative errors, and check
+    whether eq. opt_number_of_steps (integer argmin, gar_optimal_steps) picks the
+    measured-best S."""
+    import numpy as np
+    import torch
+    from scipy.optimize import nnls
+    es = 2 if dtype == "bf16" else 4
+    L = _l(P)
+    times = {}
+    for m in sizes:
+        n = max(1, m // es)
+        raw = gar_inputs.rank_inputs(P, n, dtype, ("normal", 0.0, 1.0), 77, device="cuda")
+        per16 = 16 // es
+        inp = torch.zeros((P, (n + per16 - 1) // per16 * per16), dtype=raw.dtype, device="cuda")
+        inp[:, :n] = raw          # rank rows padded to 16-byte multiples
+        del raw
+        for S in range(L, 2 * L + 1):
+            plan = gar.gar_plan_create(P, n, dtype, "sum", S)
+            gar.ensure_workspace(plan)
+            gar.gar_plan_prepare(plan, "step")
+            reps = 20 if m <= (64 << 10) else 5
+            times[(m, S)] = _time_loop(lambda: gar.gar_allreduce(plan, inp, "step", stream), reps, 3,
+                                       stream) * 1e-3
+            plan.workspace = None
+            del plan
+            torch.cuda.empty_cache()
+        del inp
+    # relative least squares (each measurement weighted by 1/t), so the microsecond
+    # small-message points count as much as the millisecond large-message ones
+    A, y = [], []
+    for (m, S), t in times.items():
+        tr, co = _paper_blocks(P, S)
+        u = m / P
+        A.append([S / t, tr * u / t, co * u / t])
+        y.append(1.0)
+    coef, _res = nnls(np.array(A), np.array(y))
+    alpha, beta, gamma = (float(c) for c in coef)
+    per = {}
+    agree = 0
+    for m in sizes:
+        meas = {S: times[(m, S)] for S in range(L, 2 * L + 1)}
+        best_meas = min(meas, key=meas.get)
+        best_model = gar.gar_optimal_steps(P, m, alpha, beta, gamma)
+        agree += int(best_meas == best_model)
+        per[str(m)] = {"measured_us": {f"S{S}": round(t * 1e6, 2) for S, t in meas.items()},
+                       "model_us": {f"S{S}": round(gar.gar_cost_model(P, S, m, alpha, beta, gamma) * 1e6, 2)
+                                    for S in meas},
+                       "measured_best_S": best_meas, "model_best_S": best_model,
+                       "model_choice_vs_best": round(meas[best_model] / meas[best_meas], 3)}
+    return {"P": P, "dtype": dtype, "mode": "step", "alpha_s": alpha, "beta_s_per_B": beta,
+            "gamma_s_per_B": gamma, "argmin_agreement": f"{agree}/{len(sizes)}", "per_size_bytes": per}
 
 
 # ---------------------------------------------------------------------------

@@ -216,6 +216,23 @@ GAR_API int gar_last_step_bytes(const gar_plan *plan, uint64_t *per_step);
 GAR_API const char *gar_strerror(int status);
 GAR_API const char *gar_last_error(void);
 
+/* The paper's cost model (Sec. "Communication model": tau = alpha + beta m + gamma m per
+ * message, blocks of u = m / P bytes) for the version with S = steps:
+ *   S = 2L (r = 0):      eq. bo_cost           2L alpha + 2(P-1) u beta + (P-1) u gamma
+ *   L < S < 2L:          eq. intemediate_cost  (2L-r) alpha + (2(P-1) + (2^r-1)(L-1)) u beta
+ *                                              + ((P-1) + (2^r-1)(2L-2)) u gamma
+ *   S = L (r = L):       eq. lo_cost           L alpha + P L u beta + P (2L-2) u gamma
+ * with L = ceil(log2 P), r = 2L - S, m_bytes = bytes per rank.  Host-only.  Returns
+ * GAR_EINVAL for P < 1 or S outside [L, 2L]. */
+GAR_API int gar_cost_model(int P, int steps, double m_bytes, double alpha, double beta,
+                           double gamma, double *tau);
+
+/* The step count minimising gar_cost_model over the integers S in [L, 2L] (eq.
+ * opt_number_of_steps gives the continuous optimum in log P; the library takes the
+ * integer argmin, smallest S on ties).  Host-only. */
+GAR_API int gar_optimal_steps(int P, double m_bytes, double alpha, double beta, double gamma,
+                              int *steps);
+
 /* Step-faithful Allreduce that allocates no device memory.  The paper has no
  * counterpart; this entry point serves callers that cannot call cudaMalloc when they
  * run an Allreduce, e.g. code whose device memory is all owned by a caching

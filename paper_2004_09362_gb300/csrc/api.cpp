@@ -2,6 +2,7 @@
 #include <cuda_runtime.h>
 
 #include <algorithm>
+#include <cmath>
 #include <cstdlib>
 #include <cstring>
 #include <new>
@@ -597,6 +598,49 @@ const char *gar_strerror(int status) {
 }
 
 const char *gar_last_error(void) { return last_error_cstr(); }
+
+int gar_cost_model(int P, int steps, double m_bytes, double alpha, double beta, double gamma,
+                   double *tau) {
+  if (P < 1 || tau == nullptr) {
+    set_error("bad cost-model arguments");
+    return GAR_EINVAL;
+  }
+  const int L = ceil_log2(P);
+  const int r = 2 * L - steps;
+  if (r < 0 || r > L) {
+    set_error("steps outside [L, 2L]");
+    return GAR_EINVAL;
+  }
+  const double u = m_bytes / P;
+  if (r == L) {  // latency-optimal, eq. lo_cost
+    *tau = L * alpha + (double)P * L * u * beta + (double)P * (2.0 * L - 2.0) * u * gamma;
+  } else {       // eq. intemediate_cost (r = 0 gives eq. bo_cost)
+    const double extra = std::ldexp(1.0, r) - 1.0;
+    *tau = (2.0 * L - r) * alpha + (2.0 * (P - 1) + extra * (L - 1)) * u * beta +
+           ((P - 1) + extra * (2.0 * L - 2.0)) * u * gamma;
+  }
+  return GAR_OK;
+}
+
+int gar_optimal_steps(int P, double m_bytes, double alpha, double beta, double gamma, int *steps) {
+  if (P < 1 || steps == nullptr) {
+    set_error("bad cost-model arguments");
+    return GAR_EINVAL;
+  }
+  const int L = ceil_log2(P);
+  int best = L;
+  double best_t = 0;
+  for (int S = L; S <= 2 * L; ++S) {
+    double t = 0;
+    gar_cost_model(P, S, m_bytes, alpha, beta, gamma, &t);
+    if (S == L || t < best_t - 1e-18) {
+      best = S;
+      best_t = t;
+    }
+  }
+  *steps = best;
+  return GAR_OK;
+}
 
 int gar_selftest_compile(void) {
   const int cases[][4] = {{24, GAR_F32, GAR_SUM, -1}, {7, GAR_F32, GAR_MAX, 3},

@@ -11,6 +11,7 @@
 #include <cuda_bf16.h>
 #include <cuda_runtime.h>
 
+#include <algorithm>
 #include <cstdint>
 #include <mutex>
 #include <string>
@@ -33,6 +34,7 @@ namespace {
 constexpr int kThreads = 256;
 constexpr uint64_t kChunk = GAR_STEP_CHUNK;  // largest chunk (elements per CTA)
 constexpr int kUnroll = GAR_STEP_UNROLL;     // 4-element vectors a thread loads at once
+constexpr uint64_t kFlatBelow = 4 * kThreads * kUnroll;  // blocks shorter than this: element-major
 
 template <int MAXP>
 struct StepArgs {
@@ -42,6 +44,7 @@ struct StepArgs {
   unsigned long long *bytes;         // counter of the communication step, or nullptr
   uint64_t q, rem, n_pad;
   uint64_t chunk;                    // elements per CTA
+  uint64_t n;                        // elements per rank
   int P, partner, nops, nchunks;
 };
 
@@ -222,6 +225,49 @@ __global__ void __launch_bounds__(kThreads) step_kernel(const __grid_constant__ 
   }
 }
 
+// Element-major form of the same launch, for small blocks: an op touches block
+// b = (x - dst_place) mod P at every rank x, i.e. every element position exactly once
+// across the P ranks, so work item g = (op, element e) maps to rank x = (b(e) + dst_place)
+// mod P.  One thread per item keeps every thread busy however short the blocks are.
+template <typename T, int OP, int MAXP>
+__global__ void __launch_bounds__(kThreads) step_kernel_flat(const __grid_constant__ StepArgs<MAXP> a) {
+  using A = typename AccOf<T>::type;
+  const uint64_t total = (uint64_t)a.nops * a.n;
+  const uint64_t big = a.rem * (a.q + 1);
+  unsigned long long moved_bytes = 0;
+  for (uint64_t g = (uint64_t)blockIdx.x * blockDim.x + threadIdx.x; g < total;
+       g += (uint64_t)gridDim.x * blockDim.x) {
+    const int oi = (int)(g / a.n);
+    const uint64_t e = g - (uint64_t)oi * a.n;
+    const StepOp op = a.ops[oi];
+    const int b = e < big ? (int)(e / (a.q + 1)) : (int)(a.rem + (e - big) / a.q);
+    const int x = (b + (int)op.dst_place) % a.P;
+    A r = A(0);
+    const bool has_recv = op.recv_place >= 0;
+    if (has_recv) {
+      const int partner = ((x + a.partner) % a.P + a.P) % a.P;
+      r = load1<T, A>(op.recv_buf, buf_ptr<A>(a, op.recv_buf, partner), e);
+      moved_bytes += (op.recv_buf == BUF_RANK) ? sizeof(T) : sizeof(A);
+    }
+    A o0 = r, o1 = r;
+    if (op.out0_own != BUF_NONE) {
+      const A v = load1<T, A>(op.out0_own, buf_ptr<A>(a, op.out0_own, x), e);
+      o0 = has_recv ? combine<OP>(v, r) : v;
+    }
+    if (op.out1_buf != BUF_NONE && op.out1_own != BUF_NONE) {
+      const A v = load1<T, A>(op.out1_own, buf_ptr<A>(a, op.out1_own, x), e);
+      o1 = has_recv ? combine<OP>(v, r) : v;
+    }
+    store1<T, A>(op.out0_buf, buf_ptr<A>(a, op.out0_buf, x), e, o0);
+    if (op.out1_buf != BUF_NONE) store1<T, A>(op.out1_buf, buf_ptr<A>(a, op.out1_buf, x), e, o1);
+  }
+  if (a.bytes != nullptr) {
+#pragma unroll
+    for (int off = 16; off > 0; off >>= 1) moved_bytes += __shfl_down_sync(0xffffffffu, moved_bytes, off);
+    if ((threadIdx.x & 31) == 0 && moved_bytes) atomicAdd(a.bytes, moved_bytes);
+  }
+}
+
 int num_sms() {
   static int sms = 0;
   if (sms == 0) {
@@ -256,10 +302,21 @@ int launch_typed(const gar_plan &pl, const Launch &ln, int launch_index, void *c
   a.q = pl.q;
   a.rem = pl.rem;
   a.n_pad = pl.n_pad;
+  a.n = pl.n;
   a.P = pl.P;
   a.partner = ln.partner;
   a.nops = ln.nops;
   const uint64_t maxblk = pl.q + (pl.rem ? 1 : 0);
+  if (maxblk < kFlatBelow && ln.nops > 0 && pl.n > 0) {
+    // blocks shorter than one CTA's worth of vectors: element-major launch
+    const uint64_t total = (uint64_t)ln.nops * pl.n;
+    const uint64_t grid = std::min<uint64_t>((total + kThreads - 1) / kThreads,
+                                             (uint64_t)num_sms() * 32);
+    step_kernel_flat<T, OP, MAXP><<<(unsigned)grid, kThreads, 0, (cudaStream_t)stream>>>(a);
+    cudaError_t e = cudaGetLastError();
+    if (e != cudaSuccess) return cuda_fail(e, "step kernel launch");
+    return GAR_OK;
+  }
   a.chunk = kChunk;
   const uint64_t min_ctas = 4 * (uint64_t)num_sms();
   while (a.chunk > 4096 && ((maxblk + a.chunk - 1) / a.chunk) * pl.P * ln.nops < min_ctas) a.chunk /= 2;

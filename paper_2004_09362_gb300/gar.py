@@ -35,6 +35,7 @@ EXPORTS = (
     "gar_plan_set_workspace", "gar_plan_compile", "gar_plan_prepare", "gar_allreduce",
     "gar_allreduce_host", "gar_allreduce_batched", "gar_last_step_bytes", "gar_strerror",
     "gar_last_error", "gar_selftest_compile", "gar_allreduce_noalloc", "gar_plan_fused_source",
+    "gar_cost_model", "gar_optimal_steps",
 )
 
 
@@ -79,6 +80,10 @@ def _load():
         "gar_selftest_compile": (i32, []),
         "gar_allreduce_noalloc": (i32, [vp, P_(vp), vp]),
         "gar_plan_fused_source": (i32, [vp, ctypes.c_char_p, P_(sz)]),
+        "gar_cost_model": (i32, [i32, i32, ctypes.c_double, ctypes.c_double, ctypes.c_double,
+                                 ctypes.c_double, P_(ctypes.c_double)]),
+        "gar_optimal_steps": (i32, [i32, ctypes.c_double, ctypes.c_double, ctypes.c_double,
+                                    ctypes.c_double, P_(i32)]),
     }
     for name, (res, args) in sig.items():
         fn = getattr(lib, name)
@@ -328,6 +333,21 @@ def gar_last_step_bytes(plan: Plan) -> list[int]:
     per = (ctypes.c_uint64 * max(1, S))()
     _check(_lib.gar_last_step_bytes(plan.handle, per), "gar_last_step_bytes")
     return [int(per[t]) for t in range(S)]
+
+
+def gar_cost_model(P: int, steps: int, m_bytes: float, alpha: float, beta: float,
+                   gamma: float) -> float:
+    t = ctypes.c_double()
+    _check(_lib.gar_cost_model(int(P), int(steps), float(m_bytes), float(alpha), float(beta),
+                               float(gamma), ctypes.byref(t)), "gar_cost_model")
+    return t.value
+
+
+def gar_optimal_steps(P: int, m_bytes: float, alpha: float, beta: float, gamma: float) -> int:
+    S = ctypes.c_int()
+    _check(_lib.gar_optimal_steps(int(P), float(m_bytes), float(alpha), float(beta), float(gamma),
+                                  ctypes.byref(S)), "gar_optimal_steps")
+    return S.value
 
 
 def gar_selftest_compile() -> None:

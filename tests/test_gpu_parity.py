@@ -94,6 +94,22 @@ def test_small_every_step_count(P, mode):
             _assert_same(got, want, dtype, f"P={P} n={n} {dtype} S={S} {mode}")
 
 
+@pytest.mark.parametrize("P", [3, 7, 12])
+def test_mid_size_chunked_step_kernel(P):
+    """Blocks of ~5000 elements with ragged starts: the chunked step-faithful launch
+    (several chunks per block, 16-byte head/tail handling), every step count and type."""
+    n = P * 5003 + 5
+    for dtype in ("f32", "i32", "bf16"):
+        t = _np_inputs(P, n, dtype, seed=33 * P)
+        host = _to_host_list(t, dtype)
+        for S in _Ss(P):
+            plan = gar.gar_plan_create(P, n, dtype, "sum", S)
+            _assert_same(_run(plan, t, "step"), G.allreduce(host, S, "sum", dtype), dtype,
+                         f"P={P} {dtype} S={S}")
+            rec = gar.gar_last_step_bytes(plan)
+            assert rec == gar.gar_plan_bytes(plan)[1]
+
+
 @pytest.mark.parametrize("op", ["max", "min"])
 @pytest.mark.parametrize("mode", ["fused", "step"])
 def test_small_max_min(op, mode):

@@ -260,3 +260,21 @@ def test_generated_source_compiles_for_config_shapes():
         plan = gar.gar_plan_create(P, n, dt, "sum", S)
         gar.gar_plan_compile(plan, "fused")
         assert plan.info()["fused_width"] >= 1
+
+
+def test_cost_model_matches_oracle():
+    """gar_cost_model / gar_optimal_steps against the oracle's restatement of eqs.
+    bo_cost, intemediate_cost, lo_cost and opt_number_of_steps (the oracle's version is
+    pinned to the paper's P=127, m=9 KiB example in test_oracle_pins)."""
+    import itertools
+    params = [(3e-5, 1e-8, 2e-10), (2.5e-6, 1.6e-13, 3e-13), (1e-6, 1e-10, 0.0), (5e-6, 0.0, 1e-12)]
+    for P in list(range(1, 40)) + [63, 64, 127, 128, 200]:
+        L = G.ceil_log2(P)
+        for m in (425.0, 9 * 1024.0, 2 ** 20, 64 * 2 ** 20):
+            for (a, b, c) in params:
+                for S in range(L, 2 * L + 1):
+                    assert gar.gar_cost_model(P, S, m, a, b, c) == pytest.approx(
+                        G.cost_model_time(P, m, S, a, b, c), rel=1e-12, abs=1e-300)
+                assert gar.gar_optimal_steps(P, m, a, b, c) == G.optimal_steps(P, m, a, b, c)
+    with pytest.raises(gar.GarError):
+        gar.gar_cost_model(8, 2, 1.0, 1.0, 1.0, 1.0)
