@@ -61,8 +61,14 @@ enum { GAR_SUM = 0, GAR_MAX = 1, GAR_MIN = 2 };
  *   gar_plan_bytes; records the bytes read from partners per step.
  * GAR_FUSED: one launch for the whole Allreduce; per element position the P
  *   contributions are loaded once, the reduction program that the schedule induces
- *   runs in registers, and every rank's result is written once. */
-enum { GAR_STEP_FAITHFUL = 0, GAR_FUSED = 1 };
+ *   runs in registers, and every rank's result is written once.
+ * GAR_STEP_PERSISTENT: the step-faithful schedule in one cooperative launch; a
+ *   grid-wide barrier separates the steps instead of a kernel boundary.  Every barrier
+ *   wait is bounded (gar_plan_debug_barrier): a CTA that waits too long records a
+ *   timeout and returns, every other CTA stops at its next poll, and
+ *   gar_plan_status reports GAR_ETIMEOUT.  Same workspace and results as
+ *   GAR_STEP_FAITHFUL. */
+enum { GAR_STEP_FAITHFUL = 0, GAR_FUSED = 1, GAR_STEP_PERSISTENT = 2 };
 
 /* Special values for the `steps` argument of gar_plan_create. */
 #define GAR_STEPS_BO (-1) /* 2 ceil(log2 P): bandwidth-optimal */
@@ -78,7 +84,8 @@ enum {
   GAR_ECUDA = -4,   /* a CUDA runtime call failed (detail in gar_last_error) */
   GAR_EJIT = -5,    /* run-time compilation of a specialized kernel failed */
   GAR_ENOWS = -6,   /* step-faithful mode needs a workspace that was not set or is too small */
-  GAR_ESTATE = -7   /* operation not valid in the plan's current state */
+  GAR_ESTATE = -7,  /* operation not valid in the plan's current state */
+  GAR_ETIMEOUT = -8 /* a bounded wait inside a kernel gave up (gar_plan_status) */
 };
 
 /* Describes a plan.  Symbols follow the paper: L = ceil(log2 P) reduction steps
@@ -207,6 +214,19 @@ typedef struct {
  * kernel's vector width fall back to element-wise loads inside the same kernel. */
 GAR_API int gar_allreduce_batched(gar_plan *const *plans, int nplans, const gar_batch_desc *desc,
                           int count, gar_stream_t stream);
+
+/* Outcome of the plan's most recent GAR_STEP_PERSISTENT Allreduce: waits for the stream
+ * it ran on, then returns GAR_OK, GAR_ETIMEOUT if a grid-barrier wait gave up (the
+ * results are then incomplete), or GAR_ECUDA.  GAR_OK if no persistent call ran. */
+GAR_API int gar_plan_status(gar_plan *plan);
+
+/* Barrier parameters of GAR_STEP_PERSISTENT.  spin_limit: polls (each an L2 round trip
+ * plus a 64 ns sleep) a CTA makes at a grid barrier before it gives up (0 restores the
+ * default, 2^20, roughly a second).
+ * phantom: extra arrivals the barrier waits for beyond the launched CTAs -- nonzero
+ * values make every wait run out, which tests the timeout path without faulting
+ * anything; keep 0 otherwise. */
+GAR_API int gar_plan_debug_barrier(gar_plan *plan, unsigned int phantom, unsigned int spin_limit);
 
 /* Bytes each communication step of the most recent step-faithful Allreduce read from
  * partner ranks, as counted by the kernels (S entries).  Synchronizes with the stream

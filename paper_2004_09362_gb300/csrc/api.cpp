@@ -36,7 +36,7 @@ int check_plan(const gar_plan *pl) {
 }
 
 int check_mode(int mode) {
-  if (mode != GAR_STEP_FAITHFUL && mode != GAR_FUSED) {
+  if (mode != GAR_STEP_FAITHFUL && mode != GAR_FUSED && mode != GAR_STEP_PERSISTENT) {
     set_error("unknown mode");
     return GAR_EINVAL;
   }
@@ -64,6 +64,20 @@ int prepare_step_faithful(gar_plan *pl) {
     e = cudaMemcpy(pl->d_ops, pl->ops.data(), pl->ops.size() * sizeof(StepOp),
                    cudaMemcpyHostToDevice);
     if (e != cudaSuccess) return cuda_fail(e, "cudaMemcpy(op table)");
+  }
+  if (pl->d_launches == nullptr && !pl->launches.empty()) {
+    std::vector<LaunchDesc> ld;
+    for (const Launch &ln : pl->launches) ld.push_back({ln.first_op, ln.nops, ln.partner, ln.comm_step});
+    cudaError_t e = cudaMalloc(&pl->d_launches, ld.size() * sizeof(LaunchDesc));
+    if (e != cudaSuccess) return cuda_fail(e, "cudaMalloc(launch table)");
+    e = cudaMemcpy(pl->d_launches, ld.data(), ld.size() * sizeof(LaunchDesc), cudaMemcpyHostToDevice);
+    if (e != cudaSuccess) return cuda_fail(e, "cudaMemcpy(launch table)");
+  }
+  if (pl->d_barrier == nullptr) {
+    cudaError_t e = cudaMalloc(&pl->d_barrier, barrier_state_bytes());
+    if (e != cudaSuccess) return cuda_fail(e, "cudaMalloc(barrier state)");
+    e = cudaMemset(pl->d_barrier, 0, barrier_state_bytes());
+    if (e != cudaSuccess) return cuda_fail(e, "cudaMemset(barrier state)");
   }
   if (pl->d_step_bytes == nullptr && pl->S > 0) {
     cudaError_t e = cudaMalloc(&pl->d_step_bytes, pl->S * sizeof(unsigned long long));
@@ -246,7 +260,7 @@ int run_host_pipelined(gar_plan *pl, const void *const *host_in, void *const *ho
   return GAR_OK;
 }
 
-int run_step_faithful(gar_plan *pl, void *const *rank, gar_stream_t stream) {
+int run_step_faithful(gar_plan *pl, void *const *rank, gar_stream_t stream, bool persistent) {
   int rc = prepare_step_faithful(pl);
   if (rc) return rc;
   if (pl->ws_bytes > 0) {
@@ -259,9 +273,17 @@ int run_step_faithful(gar_plan *pl, void *const *rank, gar_stream_t stream) {
   cudaError_t e = cudaMemsetAsync(pl->d_step_bytes, 0, pl->S * sizeof(unsigned long long),
                                   (cudaStream_t)stream);
   if (e != cudaSuccess) return cuda_fail(e, "cudaMemsetAsync(step counters)");
-  for (size_t li = 0; li < pl->launches.size(); ++li) {
-    rc = launch_step(*pl, pl->launches[li], (int)li, rank, stream);
+  if (persistent) {
+    e = cudaMemsetAsync(pl->d_barrier, 0, barrier_state_bytes(), (cudaStream_t)stream);
+    if (e != cudaSuccess) return cuda_fail(e, "cudaMemsetAsync(barrier state)");
+    rc = launch_persistent(*pl, rank, stream);
     if (rc) return rc;
+    pl->ran_persistent = true;
+  } else {
+    for (size_t li = 0; li < pl->launches.size(); ++li) {
+      rc = launch_step(*pl, pl->launches[li], (int)li, rank, stream);
+      if (rc) return rc;
+    }
   }
   pl->last_stream = stream;
   pl->ran_step_faithful = true;
@@ -325,6 +347,8 @@ void gar_plan_destroy(gar_plan *pl) {
   if (pl == nullptr) return;
   if (pl->d_ops) cudaFree(pl->d_ops);
   if (pl->d_step_bytes) cudaFree(pl->d_step_bytes);
+  if (pl->d_launches) cudaFree(pl->d_launches);
+  if (pl->d_barrier) cudaFree(pl->d_barrier);
   if (pl->hp_ready) {
     for (int k = 0; k < 3; ++k) cudaStreamDestroy((cudaStream_t)pl->hp_stream[k]);
     for (int c = 0; c < GAR_HOST_CHUNKS_MAX; ++c) {
@@ -472,8 +496,8 @@ int gar_allreduce(gar_plan *pl, void *const *rank_buffers, int mode, gar_stream_
   if (int rc = check_mode(mode)) return rc;
   if (int rc = check_buffers(pl, rank_buffers)) return rc;
   if (pl->n == 0 || pl->P == 1) return GAR_OK;
-  return mode == GAR_FUSED ? run_fused(pl, rank_buffers, stream)
-                           : run_step_faithful(pl, rank_buffers, stream);
+  if (mode == GAR_FUSED) return run_fused(pl, rank_buffers, stream);
+  return run_step_faithful(pl, rank_buffers, stream, mode == GAR_STEP_PERSISTENT);
 }
 
 int gar_allreduce_host(gar_plan *pl, const void *const *host_in, void *const *host_out,
@@ -583,6 +607,29 @@ int gar_last_step_bytes(const gar_plan *pl, uint64_t *per_step) {
   return GAR_OK;
 }
 
+int gar_plan_status(gar_plan *pl) {
+  if (int rc = check_plan(pl)) return rc;
+  if (!pl->ran_persistent || pl->d_barrier == nullptr) return GAR_OK;
+  cudaError_t e = cudaStreamSynchronize((cudaStream_t)pl->last_stream);
+  if (e != cudaSuccess) return cuda_fail(e, "cudaStreamSynchronize");
+  int st[4] = {0, 0, 0, 0};
+  e = cudaMemcpy(st, pl->d_barrier, sizeof st, cudaMemcpyDeviceToHost);
+  if (e != cudaSuccess) return cuda_fail(e, "cudaMemcpy(barrier state)");
+  if (st[2] != 0) {
+    set_error("persistent step-faithful kernel: a grid-barrier wait gave up after launch " +
+              std::to_string(st[3]));
+    return GAR_ETIMEOUT;
+  }
+  return GAR_OK;
+}
+
+int gar_plan_debug_barrier(gar_plan *pl, unsigned int phantom, unsigned int spin_limit) {
+  if (int rc = check_plan(pl)) return rc;
+  pl->barrier_phantom = phantom;
+  pl->barrier_spin_limit = spin_limit ? spin_limit : (1u << 20);
+  return GAR_OK;
+}
+
 const char *gar_strerror(int status) {
   switch (status) {
     case GAR_OK: return "success";
@@ -593,6 +640,7 @@ const char *gar_strerror(int status) {
     case GAR_EJIT: return "kernel compilation failed";
     case GAR_ENOWS: return "workspace missing or too small";
     case GAR_ESTATE: return "invalid plan state";
+    case GAR_ETIMEOUT: return "bounded wait timed out";
   }
   return "unknown status";
 }

@@ -44,6 +44,11 @@ struct Launch {
   int nops;
 };
 
+// Launch descriptor as the persistent kernel reads it from device memory.
+struct LaunchDesc {
+  int first_op, nops, partner, comm_step;
+};
+
 struct CommStep {
   int phase;                      // 0 reduce, 1 distribute
   int i;                          // the paper's step index i
@@ -91,6 +96,12 @@ struct gar_plan {
   bool ran_step_faithful = false;
   gar::JitKernel *fused = nullptr;   // owned by the JIT cache
   int fused_width = 0;
+  // persistent step-faithful mode: launch table, barrier state, barrier parameters
+  void *d_launches = nullptr;
+  void *d_barrier = nullptr;
+  unsigned int barrier_spin_limit = 1u << 20;   // polls: ~0.5-1 s (each is an L2 round trip + 64 ns)
+  unsigned int barrier_phantom = 0;
+  bool ran_persistent = false;
   // pipelined host-buffer path: 3 streams (to device, kernel, to host) and events
   bool hp_ready = false;
   void *hp_stream[3] = {nullptr, nullptr, nullptr};
@@ -135,6 +146,8 @@ int jit_load(JitKernel *k);
 // step_kernels.cu
 int launch_step(const gar_plan &pl, const Launch &ln, int launch_index, void *const *rank,
                 gar_stream_t stream);
+int launch_persistent(const gar_plan &pl, void *const *rank, gar_stream_t stream);
+size_t barrier_state_bytes();
 
 // api.cpp
 void set_error(const std::string &msg);

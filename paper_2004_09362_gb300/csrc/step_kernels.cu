@@ -132,26 +132,34 @@ __device__ __forceinline__ void *buf_ptr(const StepArgs<MAXP> &a, uint8_t buf, i
   return static_cast<char *>(a.ws[buf - BUF_QP0]) + (uint64_t)rank * a.n_pad * sizeof(A);
 }
 
+// Per-launch parameters the work functions need besides the buffers.
+struct LaunchView {
+  const StepOp *ops;
+  unsigned long long *bytes;  // counter of the communication step, or nullptr
+  uint64_t chunk;             // elements per CTA item (chunked mapping)
+  int nops, partner, nchunks;
+};
+
+// Chunked mapping: work item `item` = (chunk, rank x, op) is done by the whole CTA.
 template <typename T, int OP, int MAXP>
-__global__ void __launch_bounds__(kThreads) step_kernel(const __grid_constant__ StepArgs<MAXP> a) {
+__device__ __forceinline__ void chunk_work(const StepArgs<MAXP> &a, const LaunchView &lv, uint64_t item) {
   using A = typename AccOf<T>::type;
-  uint64_t bid = blockIdx.x;
-  const int chunk = (int)(bid % (uint64_t)a.nchunks);
-  bid /= (uint64_t)a.nchunks;
-  const int x = (int)(bid % (uint64_t)a.P);
-  const int oi = (int)(bid / (uint64_t)a.P);
-  if (oi >= a.nops) return;
-  const StepOp op = a.ops[oi];
+  const int chunk = (int)(item % (uint64_t)lv.nchunks);
+  item /= (uint64_t)lv.nchunks;
+  const int x = (int)(item % (uint64_t)a.P);
+  const int oi = (int)(item / (uint64_t)a.P);
+  if (oi >= lv.nops) return;
+  const StepOp op = lv.ops[oi];
   const int b = ((x - (int)op.dst_place) % a.P + a.P) % a.P;
   const uint64_t bstart = (uint64_t)b * a.q + ((uint64_t)b < a.rem ? (uint64_t)b : a.rem);
   const uint64_t blen = a.q + ((uint64_t)b < a.rem ? 1 : 0);
-  const uint64_t c0 = (uint64_t)chunk * a.chunk;
+  const uint64_t c0 = (uint64_t)chunk * lv.chunk;
   if (c0 >= blen) return;
   const uint64_t lo = bstart + c0;
-  const uint64_t hi = bstart + (blen < c0 + a.chunk ? blen : c0 + a.chunk);
+  const uint64_t hi = bstart + (blen < c0 + lv.chunk ? blen : c0 + lv.chunk);
 
   const bool has_recv = op.recv_place >= 0;
-  const int partner = ((x + a.partner) % a.P + a.P) % a.P;
+  const int partner = ((x + lv.partner) % a.P + a.P) % a.P;
   const void *recv = has_recv ? buf_ptr<A>(a, op.recv_buf, partner) : nullptr;
   void *out0 = buf_ptr<A>(a, op.out0_buf, x);
   const void *own0 = buf_ptr<A>(a, op.out0_own, x);
@@ -216,36 +224,37 @@ __global__ void __launch_bounds__(kThreads) step_kernel(const __grid_constant__ 
   for (uint64_t e = va + 4 * (uint64_t)threadIdx.x; e < vb; e += kUnroll * vstride) do4xU(e, vstride, vb);
   for (uint64_t e = vb + threadIdx.x; e < hi; e += blockDim.x) do1(e);
 
-  if (a.bytes != nullptr && has_recv) {
+  if (lv.bytes != nullptr && has_recv) {
     unsigned long long m = moved;
 #pragma unroll
     for (int off = 16; off > 0; off >>= 1) m += __shfl_down_sync(0xffffffffu, m, off);
     const unsigned long long esize = (op.recv_buf == BUF_RANK) ? sizeof(T) : sizeof(A);
-    if ((threadIdx.x & 31) == 0 && m) atomicAdd(a.bytes, m * esize);
+    if ((threadIdx.x & 31) == 0 && m) atomicAdd(lv.bytes, m * esize);
   }
 }
 
-// Element-major form of the same launch, for small blocks: an op touches block
-// b = (x - dst_place) mod P at every rank x, i.e. every element position exactly once
-// across the P ranks, so work item g = (op, element e) maps to rank x = (b(e) + dst_place)
-// mod P.  One thread per item keeps every thread busy however short the blocks are.
+// Element-major mapping, for small blocks: an op touches block b = (x - dst_place) mod P
+// at every rank x, i.e. every element position exactly once across the P ranks, so
+// work item g = (op, element e) maps to rank x = (b(e) + dst_place) mod P.  One thread
+// per item keeps every thread busy however short the blocks are.  Threads g_first,
+// g_first + g_stride, ... of the launch's nops * n items.
 template <typename T, int OP, int MAXP>
-__global__ void __launch_bounds__(kThreads) step_kernel_flat(const __grid_constant__ StepArgs<MAXP> a) {
+__device__ __forceinline__ void flat_work(const StepArgs<MAXP> &a, const LaunchView &lv, uint64_t g_first,
+                                          uint64_t g_stride) {
   using A = typename AccOf<T>::type;
-  const uint64_t total = (uint64_t)a.nops * a.n;
+  const uint64_t total = (uint64_t)lv.nops * a.n;
   const uint64_t big = a.rem * (a.q + 1);
   unsigned long long moved_bytes = 0;
-  for (uint64_t g = (uint64_t)blockIdx.x * blockDim.x + threadIdx.x; g < total;
-       g += (uint64_t)gridDim.x * blockDim.x) {
+  for (uint64_t g = g_first; g < total; g += g_stride) {
     const int oi = (int)(g / a.n);
     const uint64_t e = g - (uint64_t)oi * a.n;
-    const StepOp op = a.ops[oi];
+    const StepOp op = lv.ops[oi];
     const int b = e < big ? (int)(e / (a.q + 1)) : (int)(a.rem + (e - big) / a.q);
     const int x = (b + (int)op.dst_place) % a.P;
     A r = A(0);
     const bool has_recv = op.recv_place >= 0;
     if (has_recv) {
-      const int partner = ((x + a.partner) % a.P + a.P) % a.P;
+      const int partner = ((x + lv.partner) % a.P + a.P) % a.P;
       r = load1<T, A>(op.recv_buf, buf_ptr<A>(a, op.recv_buf, partner), e);
       moved_bytes += (op.recv_buf == BUF_RANK) ? sizeof(T) : sizeof(A);
     }
@@ -261,10 +270,130 @@ __global__ void __launch_bounds__(kThreads) step_kernel_flat(const __grid_consta
     store1<T, A>(op.out0_buf, buf_ptr<A>(a, op.out0_buf, x), e, o0);
     if (op.out1_buf != BUF_NONE) store1<T, A>(op.out1_buf, buf_ptr<A>(a, op.out1_buf, x), e, o1);
   }
-  if (a.bytes != nullptr) {
+  if (lv.bytes != nullptr) {
 #pragma unroll
     for (int off = 16; off > 0; off >>= 1) moved_bytes += __shfl_down_sync(0xffffffffu, moved_bytes, off);
-    if ((threadIdx.x & 31) == 0 && moved_bytes) atomicAdd(a.bytes, moved_bytes);
+    if ((threadIdx.x & 31) == 0 && moved_bytes) atomicAdd(lv.bytes, moved_bytes);
+  }
+}
+
+template <int MAXP>
+__device__ __forceinline__ LaunchView view_of(const StepArgs<MAXP> &a) {
+  LaunchView lv;
+  lv.ops = a.ops;
+  lv.bytes = a.bytes;
+  lv.chunk = a.chunk;
+  lv.nops = a.nops;
+  lv.partner = a.partner;
+  lv.nchunks = a.nchunks;
+  return lv;
+}
+
+template <typename T, int OP, int MAXP>
+__global__ void __launch_bounds__(kThreads) step_kernel(const __grid_constant__ StepArgs<MAXP> a) {
+  chunk_work<T, OP, MAXP>(a, view_of(a), blockIdx.x);
+}
+
+template <typename T, int OP, int MAXP>
+__global__ void __launch_bounds__(kThreads) step_kernel_flat(const __grid_constant__ StepArgs<MAXP> a) {
+  flat_work<T, OP, MAXP>(a, view_of(a), (uint64_t)blockIdx.x * blockDim.x + threadIdx.x,
+                         (uint64_t)gridDim.x * blockDim.x);
+}
+
+// ---------------------------------------------------------------------------
+// Persistent step-faithful mode (GAR_STEP_PERSISTENT): one cooperative launch runs every
+// step of the schedule; a grid-wide barrier between steps takes the place of the kernel
+// boundary.  The barrier's waits are bounded: after spin_limit polls a CTA records a
+// timeout in the barrier state and returns, and every other CTA stops at its next poll,
+// so the kernel always ends and the context stays usable; the host reads the outcome
+// with gar_plan_status.
+// ---------------------------------------------------------------------------
+
+struct BarrierState {
+  unsigned int count;   // arrivals at the current barrier
+  unsigned int gen;     // barrier generation
+  int error;            // 1 once any CTA gave up waiting
+  int error_launch;     // launch index after which the first timeout happened
+};
+
+template <int MAXP>
+struct PersistArgs {
+  StepArgs<MAXP> s;                 // buffers and sizes (s.ops = whole op table)
+  const LaunchDesc *launches;
+  unsigned long long *step_bytes;   // per communication step, or nullptr
+  BarrierState *bar;
+  int nlaunch;
+  int flat;                         // element-major mapping (small blocks)
+  unsigned int spin_limit;          // polls before a wait gives up
+  unsigned int phantom;             // arrivals expected beyond the grid (test hook, normally 0)
+};
+
+__device__ __forceinline__ unsigned ld_acquire_gpu(const unsigned *p) {
+  unsigned v;
+  asm volatile("ld.acquire.gpu.global.u32 %0, [%1];" : "=r"(v) : "l"(p) : "memory");
+  return v;
+}
+__device__ __forceinline__ void st_release_gpu(unsigned *p, unsigned v) {
+  asm volatile("st.release.gpu.global.u32 [%0], %1;" ::"l"(p), "r"(v) : "memory");
+}
+__device__ __forceinline__ int ld_relaxed_int(const int *p) {
+  int v;
+  asm volatile("ld.relaxed.gpu.global.s32 %0, [%1];" : "=r"(v) : "l"(p) : "memory");
+  return v;
+}
+
+// Grid-wide barrier with a bounded wait.  Returns false (for the whole CTA) if this or
+// any other CTA timed out.
+__device__ bool grid_barrier(BarrierState *bar, unsigned expected, unsigned spin_limit, int launch) {
+  __shared__ int s_ok;
+  __syncthreads();  // every thread's writes of this step precede thread 0's fence
+  if (threadIdx.x == 0) {
+    int ok = 1;
+    const unsigned g = ld_acquire_gpu(&bar->gen);
+    __threadfence();
+    const unsigned arrived = atomicAdd(&bar->count, 1u) + 1u;
+    if (arrived == expected) {
+      atomicExch(&bar->count, 0u);
+      __threadfence();
+      st_release_gpu(&bar->gen, g + 1u);
+    } else {
+      unsigned polls = 0;
+      while (ld_acquire_gpu(&bar->gen) == g) {
+        if (++polls >= spin_limit || ld_relaxed_int(&bar->error) != 0) {
+          ok = 0;
+          break;
+        }
+        __nanosleep(64);
+      }
+    }
+    if (!ok && atomicCAS(&bar->error, 0, 1) == 0) bar->error_launch = launch;
+    __threadfence();
+    s_ok = ok;
+  }
+  __syncthreads();
+  return s_ok != 0;
+}
+
+template <typename T, int OP, int MAXP>
+__global__ void __launch_bounds__(kThreads) step_kernel_persistent(const __grid_constant__ PersistArgs<MAXP> p) {
+  const unsigned expected = gridDim.x + p.phantom;
+  for (int l = 0; l < p.nlaunch; ++l) {
+    const LaunchDesc d = p.launches[l];
+    LaunchView lv;
+    lv.ops = p.s.ops + d.first_op;
+    lv.nops = d.nops;
+    lv.partner = d.partner;
+    lv.bytes = (p.step_bytes != nullptr && d.comm_step >= 0) ? p.step_bytes + d.comm_step : nullptr;
+    lv.chunk = p.s.chunk;
+    lv.nchunks = p.s.nchunks;
+    if (p.flat) {
+      flat_work<T, OP, MAXP>(p.s, lv, (uint64_t)blockIdx.x * blockDim.x + threadIdx.x,
+                             (uint64_t)gridDim.x * blockDim.x);
+    } else {
+      const uint64_t items = (uint64_t)lv.nchunks * (uint64_t)p.s.P * (uint64_t)lv.nops;
+      for (uint64_t item = blockIdx.x; item < items; item += gridDim.x) chunk_work<T, OP, MAXP>(p.s, lv, item);
+    }
+    if (l + 1 < p.nlaunch && !grid_barrier(p.bar, expected, p.spin_limit, l)) return;
   }
 }
 
@@ -353,6 +482,63 @@ int launch_dt(const gar_plan &pl, const Launch &ln, int li, void *const *rank, g
   return GAR_EINVAL;
 }
 
+template <typename T, int OP, int MAXP>
+int launch_persistent_typed(const gar_plan &pl, void *const *rank, gar_stream_t stream) {
+  PersistArgs<MAXP> p{};
+  for (int x = 0; x < pl.P; ++x) p.s.rank[x] = rank[x];
+  int slot = 0;
+  for (int k = 0; k < NUM_WS_BUFS; ++k)
+    p.s.ws[k] = pl.ws_used[k] ? static_cast<char *>(pl.ws) + (size_t)(slot++) * pl.P * pl.n_pad * acc_size(pl.dtype)
+                              : nullptr;
+  p.s.ops = pl.d_ops;
+  p.s.bytes = nullptr;
+  p.s.q = pl.q;
+  p.s.rem = pl.rem;
+  p.s.n_pad = pl.n_pad;
+  p.s.n = pl.n;
+  p.s.P = pl.P;
+  const uint64_t maxblk = pl.q + (pl.rem ? 1 : 0);
+  p.flat = maxblk < kFlatBelow ? 1 : 0;
+  p.s.chunk = kChunk;
+  p.s.nchunks = (int)((maxblk + kChunk - 1) / kChunk);
+  p.launches = static_cast<const LaunchDesc *>(pl.d_launches);
+  p.step_bytes = pl.d_step_bytes;
+  p.bar = static_cast<BarrierState *>(pl.d_barrier);
+  p.nlaunch = (int)pl.launches.size();
+  p.spin_limit = pl.barrier_spin_limit;
+  p.phantom = pl.barrier_phantom;
+  const void *fn = (const void *)step_kernel_persistent<T, OP, MAXP>;
+  int per_sm = 0;
+  cudaError_t e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, fn, kThreads, 0);
+  if (e != cudaSuccess || per_sm < 1) return cuda_fail(e == cudaSuccess ? cudaErrorInvalidConfiguration : e,
+                                                       "persistent kernel occupancy");
+  const unsigned grid = (unsigned)(per_sm * num_sms());
+  void *args[] = {&p};
+  e = cudaLaunchCooperativeKernel(fn, dim3(grid), dim3(kThreads), args, 0, (cudaStream_t)stream);
+  if (e != cudaSuccess) return cuda_fail(e, "persistent kernel launch");
+  return GAR_OK;
+}
+
+template <typename T, int MAXP>
+int launch_persistent_op(const gar_plan &pl, void *const *rank, gar_stream_t s) {
+  switch (pl.op) {
+    case GAR_SUM: return launch_persistent_typed<T, GAR_SUM, MAXP>(pl, rank, s);
+    case GAR_MAX: return launch_persistent_typed<T, GAR_MAX, MAXP>(pl, rank, s);
+    case GAR_MIN: return launch_persistent_typed<T, GAR_MIN, MAXP>(pl, rank, s);
+  }
+  return GAR_EINVAL;
+}
+
+template <int MAXP>
+int launch_persistent_dt(const gar_plan &pl, void *const *rank, gar_stream_t s) {
+  switch (pl.dtype) {
+    case GAR_F32: return launch_persistent_op<float, MAXP>(pl, rank, s);
+    case GAR_BF16: return launch_persistent_op<__nv_bfloat16, MAXP>(pl, rank, s);
+    case GAR_I32: return launch_persistent_op<int, MAXP>(pl, rank, s);
+  }
+  return GAR_EINVAL;
+}
+
 }  // namespace
 
 int launch_step(const gar_plan &pl, const Launch &ln, int launch_index, void *const *rank,
@@ -360,6 +546,13 @@ int launch_step(const gar_plan &pl, const Launch &ln, int launch_index, void *co
   if (pl.P <= 128) return launch_dt<128>(pl, ln, launch_index, rank, stream);
   return launch_dt<GAR_MAX_P>(pl, ln, launch_index, rank, stream);
 }
+
+int launch_persistent(const gar_plan &pl, void *const *rank, gar_stream_t stream) {
+  if (pl.P <= 128) return launch_persistent_dt<128>(pl, rank, stream);
+  return launch_persistent_dt<GAR_MAX_P>(pl, rank, stream);
+}
+
+size_t barrier_state_bytes() { return sizeof(BarrierState); }
 
 }  // namespace gar
 

@@ -18,14 +18,15 @@ _LIB_PATH = os.path.join(_HERE, "libgar.so")
 
 GAR_F32, GAR_BF16, GAR_I32 = 0, 1, 2
 GAR_SUM, GAR_MAX, GAR_MIN = 0, 1, 2
-GAR_STEP_FAITHFUL, GAR_FUSED = 0, 1
+GAR_STEP_FAITHFUL, GAR_FUSED, GAR_STEP_PERSISTENT = 0, 1, 2
 GAR_STEPS_BO, GAR_STEPS_LO = -1, -2
 GAR_MAX_P = 1024
 GAR_OK = 0
 
 DTYPES = {"f32": GAR_F32, "bf16": GAR_BF16, "i32": GAR_I32}
 OPS = {"sum": GAR_SUM, "max": GAR_MAX, "min": GAR_MIN}
-MODES = {"step": GAR_STEP_FAITHFUL, "step_faithful": GAR_STEP_FAITHFUL, "fused": GAR_FUSED}
+MODES = {"step": GAR_STEP_FAITHFUL, "step_faithful": GAR_STEP_FAITHFUL, "fused": GAR_FUSED,
+         "persistent": GAR_STEP_PERSISTENT}
 ELEM_SIZE = {GAR_F32: 4, GAR_BF16: 2, GAR_I32: 4}
 
 # Every symbol include/gar.h declares (checked by the CPU tests).
@@ -35,7 +36,7 @@ EXPORTS = (
     "gar_plan_set_workspace", "gar_plan_compile", "gar_plan_prepare", "gar_allreduce",
     "gar_allreduce_host", "gar_allreduce_batched", "gar_last_step_bytes", "gar_strerror",
     "gar_last_error", "gar_selftest_compile", "gar_allreduce_noalloc", "gar_plan_fused_source",
-    "gar_cost_model", "gar_optimal_steps",
+    "gar_cost_model", "gar_optimal_steps", "gar_plan_status", "gar_plan_debug_barrier",
 )
 
 
@@ -84,6 +85,8 @@ def _load():
                                  ctypes.c_double, P_(ctypes.c_double)]),
         "gar_optimal_steps": (i32, [i32, ctypes.c_double, ctypes.c_double, ctypes.c_double,
                                     ctypes.c_double, P_(i32)]),
+        "gar_plan_status": (i32, [vp]),
+        "gar_plan_debug_barrier": (i32, [vp, ctypes.c_uint, ctypes.c_uint]),
     }
     for name, (res, args) in sig.items():
         fn = getattr(lib, name)
@@ -280,9 +283,22 @@ def ensure_workspace(plan: Plan, device=None):
     return plan.workspace
 
 
+def gar_plan_status(plan: Plan) -> int:
+    """GAR_OK, or the status code of the last persistent Allreduce (raises on CUDA errors)."""
+    rc = _lib.gar_plan_status(plan.handle)
+    if rc not in (GAR_OK, -8):
+        _check(rc, "gar_plan_status")
+    return rc
+
+
+def gar_plan_debug_barrier(plan: Plan, phantom: int = 0, spin_limit: int = 0) -> None:
+    _check(_lib.gar_plan_debug_barrier(plan.handle, int(phantom), int(spin_limit)),
+           "gar_plan_debug_barrier")
+
+
 def gar_allreduce(plan: Plan, rank_buffers, mode="fused", stream=None) -> None:
     mode_c = _code(mode, MODES, "mode")
-    if mode_c == GAR_STEP_FAITHFUL and plan.workspace is None:
+    if mode_c in (GAR_STEP_FAITHFUL, GAR_STEP_PERSISTENT) and plan.workspace is None:
         ensure_workspace(plan)
     ptrs = _ptr_array(rank_pointers(rank_buffers))
     _check(_lib.gar_allreduce(plan.handle, ptrs, mode_c, _stream_handle(stream)), "gar_allreduce")
@@ -290,7 +306,7 @@ def gar_allreduce(plan: Plan, rank_buffers, mode="fused", stream=None) -> None:
 
 def gar_allreduce_host(plan: Plan, host_in, host_out, dev_bufs, mode="fused", stream=None) -> None:
     mode_c = _code(mode, MODES, "mode")
-    if mode_c == GAR_STEP_FAITHFUL and plan.workspace is None:
+    if mode_c in (GAR_STEP_FAITHFUL, GAR_STEP_PERSISTENT) and plan.workspace is None:
         ensure_workspace(plan)
     hin = _ptr_array(rank_pointers(host_in))
     hout = _ptr_array(rank_pointers(host_out))

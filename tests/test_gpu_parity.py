@@ -346,6 +346,47 @@ def test_batched_mixed_order_and_steps():
 
 
 # ---------------------------------------------------------------------------
+# Persistent step-faithful mode: one cooperative launch, bounded grid barriers
+# ---------------------------------------------------------------------------
+
+@pytest.mark.parametrize("P", [2, 5, 7, 8, 13, 24, 33])
+def test_persistent_matches_oracle(P):
+    """Small blocks (element-major mapping) and mid-size blocks (chunked mapping),
+    every step count, all three types; recorded step bytes; no barrier timeout."""
+    for n in (3 * P + 1, P * 3001 + 7):
+        for dtype in ("f32", "i32", "bf16"):
+            if n > 1000 and dtype != "f32" and P not in (7, 24):
+                continue
+            t = _np_inputs(P, n, dtype, seed=5 * P + n)
+            host = _to_host_list(t, dtype)
+            for S in _Ss(P):
+                plan = gar.gar_plan_create(P, n, dtype, "sum", S)
+                got = _run(plan, t, "persistent")
+                assert gar.gar_plan_status(plan) == 0
+                _assert_same(got, G.allreduce(host, S, "sum", dtype), dtype,
+                             f"persistent P={P} n={n} {dtype} S={S}")
+                assert gar.gar_last_step_bytes(plan) == gar.gar_plan_bytes(plan)[1]
+
+
+def test_persistent_barrier_timeout_is_reported_and_recoverable():
+    """Make every grid-barrier wait run out (the barrier waits for one CTA that was never
+    launched): the kernel returns on its own, gar_plan_status reports GAR_ETIMEOUT, and
+    the same context then runs correct Allreduces."""
+    P, n, S = 7, 5000, 4
+    t = _np_inputs(P, n, "f32", seed=1)
+    plan = gar.gar_plan_create(P, n, "f32", "sum", S)
+    gar.gar_plan_debug_barrier(plan, phantom=1, spin_limit=2000)
+    _run(plan, t, "persistent")
+    assert gar.gar_plan_status(plan) == -8
+    assert "gave up" in gar.gar_last_error()
+    gar.gar_plan_debug_barrier(plan, phantom=0, spin_limit=0)
+    want = G.allreduce(_to_host_list(t, "f32"), S, "sum", "f32")
+    _assert_same(_run(plan, t, "persistent"), want, "f32", "after timeout")
+    assert gar.gar_plan_status(plan) == 0
+    _assert_same(_run(plan, t, "fused"), want, "f32", "fused after timeout")
+
+
+# ---------------------------------------------------------------------------
 # Host-buffer entry point and argument handling on the device
 # ---------------------------------------------------------------------------
 
