@@ -45,6 +45,15 @@ version", "Latency-optimal version")
   t^{+floor(N_i/2)} (end of Sec. "Bandwidth-optimal algorithm").
 * Result: process x's block b is the vector at placement (x - b) mod P.
 
+Groups: T_P is the cyclic group (Table 1a) by default.  group="xor" uses the
+self-inverse group of Table 1b (t_k(x) = x XOR k, P a power of two).  Everything above
+is written with the group operation: placement k puts block i on process t_k(i); a step
+moves the transmitted vectors by the group element that takes index k to index
+k - floor(N_i/2), which is t_{floor(N_i/2)}^{-1} (t^{-floor(N_i/2)} in the cyclic group,
+t_{N_i/2} itself in the XOR group, where k - N_i/2 = k XOR N_i/2 for the transmitted
+indices); copy s of the schedule has index k at placement t_s(k); distribution moves by
+t_{floor(N_i/2)} (reading C18).
+
 Precision: f32 runs in float32 (IEEE round-to-nearest-even, as numpy does it); i32 in
 int32 with two's-complement wraparound; bf16 inputs are widened exactly to float32,
 every partial is float32, and each q_Sigma is rounded to bf16 once, at the end of the
@@ -66,7 +75,7 @@ __all__ = [
     "OPS", "DTYPES", "ceil_log2", "vector_counts", "block_bounds", "schedule_shape",
     "ExprTable", "Run", "simulate", "allreduce", "round_to_bf16", "is_bf16_exact",
     "column_reduce_exact", "kahan_sum_f64", "tree_string", "parse_tree",
-    "eval_tree", "cost_model_time", "optimal_steps",
+    "eval_tree", "cost_model_time", "optimal_steps", "group_ops",
 ]
 
 OPS = ("sum", "max", "min")
@@ -216,16 +225,32 @@ def eval_tree(t, leaf_value, op: str):
     return _combine(op, eval_tree(t[0], leaf_value, op), eval_tree(t[1], leaf_value, op))
 
 
-def _reduce_partner(x: int, d: int, P: int) -> int:
-    """Where process x sends during a reduction step: the operator t^{-d} moves every
-    block from x to x - d (eqs. comm_op_0, bo_dir_perms)."""
-    return (x - d) % P
+def group_ops(P: int, group: str):
+    """(op, inverse) of the permutation group T_P acting on {0..P-1}: t_a(t_b(x)) =
+    op(op(x, b), a).  "cyclic": t_k(x) = x + k mod P (Table 1a); "xor": t_k(x) = x XOR k,
+    the self-inverse group generated by the h_i of Table 1b (P a power of two)."""
+    if group == "cyclic":
+        return (lambda a, b: (a + b) % P), (lambda a: (-a) % P)
+    if group == "xor":
+        if P & (P - 1):
+            raise ValueError("the XOR group (Table 1b) needs P a power of two")
+        return (lambda a, b: a ^ b), (lambda a: a)
+    raise ValueError(group)
 
 
-def _distribute_partner(x: int, d: int, P: int) -> int:
-    """Where process x sends during a distribution step: the reversed operator t^{+d}
-    (end of Sec. "Bandwidth-optimal algorithm")."""
-    return (x + d) % P
+def _reduce_partner(x: int, d: int, P: int, group: str = "cyclic") -> int:
+    """Where process x sends during a reduction step: the step operator
+    t_d^{-1} (t^{-d} in the cyclic group, eqs. comm_op_0, bo_dir_perms) moves every
+    block from x to t_d^{-1}(x)."""
+    op, inv = group_ops(P, group)
+    return op(x, inv(d))
+
+
+def _distribute_partner(x: int, d: int, P: int, group: str = "cyclic") -> int:
+    """Where process x sends during a distribution step: the reversed operator t_d
+    (t^{+d} in the cyclic group; end of Sec. "Bandwidth-optimal algorithm")."""
+    op, _inv = group_ops(P, group)
+    return op(x, d)
 
 
 def _combine(op: str, a, b):
@@ -314,7 +339,7 @@ class Run:
 
 
 def simulate(P: int, n: int, steps: int, inputs=None, op: str = "sum",
-             dtype: str = "f32", elements=None) -> Run:
+             dtype: str = "f32", elements=None, group: str = "cyclic") -> Run:
     """Run the Allreduce schedule with P explicit process stores and explicit
     per-step message lists.
 
@@ -329,6 +354,7 @@ def simulate(P: int, n: int, steps: int, inputs=None, op: str = "sum",
         raise ValueError(op)
     if dtype not in DTYPES:
         raise ValueError(dtype)
+    gop, ginv = group_ops(P, group)
     shape = schedule_shape(P, steps)
     L, r, K = shape["L"], shape["r"], shape["K"]
     Ns = vector_counts(P)
@@ -358,18 +384,19 @@ def simulate(P: int, n: int, steps: int, inputs=None, op: str = "sum",
                 raise ValueError("bf16 inputs must be exactly representable in bf16")
 
     # --- initial data: Q_initial = t_0 q_0 : t_1 q_1 : ... : t_{P-1} q_{P-1}
-    # (eq. distr_vector_set).  Process x holds block (x - k) mod P of t_k q_k, which is
-    # its own block u_{x-k, x}.
+    # (eq. distr_vector_set).  Process x holds block b = t_k^{-1}(x) of t_k q_k (block b
+    # sits on t_k(b) = x), which is its own block u_{b, x}.
     store = [dict() for _ in range(P)]
     for x in range(P):
         for k in range(P):
             key = (k, ex.leaf(k))
-            b = (x - k) % P
+            b = gop(x, ginv(k))
             store[x][key] = inputs[x][sel[b]].copy() if have_values else None
 
     # Each shifted copy s of the schedule starts from the same initial set, its index k
-    # naming the vector at placement s + k (eq. var_starting_set).
-    sched = [[((s + k) % P, ex.leaf((s + k) % P)) for k in range(P)] for s in range(K)]
+    # naming the vector at placement t_s(k) (s + k in the cyclic group; eq.
+    # var_starting_set).
+    sched = [[(gop(s, k), ex.leaf(gop(s, k))) for k in range(P)] for s in range(K)]
     run = Run(P=P, n=n, steps=steps, L=L, r=r, K=K, op=op, dtype=dtype, exprs=ex,
               outputs=None)
 
@@ -392,14 +419,14 @@ def simulate(P: int, n: int, steps: int, inputs=None, op: str = "sum",
         messages = []
         inbox = [dict() for _ in range(P)]
         for x in range(P):
-            dst = _reduce_partner(x, d, P)
+            dst = _reduce_partner(x, d, P, group)
             items = []
             for key in tx:
-                b = (x - key[0]) % P
+                b = gop(x, ginv(key[0]))
                 sz = itemsize if ex.is_leaf(key[1]) else acc_itemsize
                 items.append((key, block_len[b], sz))
-                # the block keeps its index; its placement moves by -d
-                moved = ((key[0] - d) % P, key[1])
+                # the block keeps its index; its placement moves by t_d^{-1}
+                moved = (gop(key[0], ginv(d)), key[1])
                 inbox[dst][moved] = store[x][key]
             messages.append((x, dst, items))
         run.log.append({"phase": "reduce", "i": i, "N": N, "d": d,
@@ -419,7 +446,7 @@ def simulate(P: int, n: int, steps: int, inputs=None, op: str = "sum",
                         new_store[x][key] = store[x][key]
                 else:
                     own = q[k]
-                    moved = ((q[k + d][0] - d) % P, q[k + d][1])
+                    moved = (gop(q[k + d][0], ginv(d)), q[k + d][1])
                     assert moved[0] == own[0]
                     key = (own[0], ex.pair(own[1], moved[1]))
                     if key not in combined:
@@ -458,27 +485,27 @@ def simulate(P: int, n: int, steps: int, inputs=None, op: str = "sum",
         messages = []
         inbox = [dict() for _ in range(P)]
         for x in range(P):
-            dst = _distribute_partner(x, d, P)
+            dst = _distribute_partner(x, d, P, group)
             items = []
             for p in senders:
                 key = at_place[p]
-                b = (x - p) % P
+                b = gop(x, ginv(p))
                 items.append((key, block_len[b], itemsize))
-                inbox[dst][((p + d) % P, key[1])] = store[x][key]
+                inbox[dst][(gop(p, d), key[1])] = store[x][key]
             messages.append((x, dst, items))
         run.log.append({"phase": "distribute", "i": i, "N": N, "d": d,
                         "tx": [at_place[p] for p in senders], "messages": messages})
         for p in senders:
-            newkey = ((p + d) % P, at_place[p][1])
-            assert (p + d) % P not in at_place
-            at_place[(p + d) % P] = newkey
+            newkey = (gop(p, d), at_place[p][1])
+            assert gop(p, d) not in at_place
+            at_place[gop(p, d)] = newkey
             for x in range(P):
                 store[x][newkey] = inbox[x][newkey]
 
     assert sorted(at_place) == list(range(P))
 
-    # --- result: process x's block b sits at placement (x - b) mod P
-    run.out_key = [[at_place[(x - b) % P] for b in range(P)] for x in range(P)]
+    # --- result: process x's block b sits at the placement p with t_p(b) = x
+    run.out_key = [[at_place[gop(x, ginv(b))] for b in range(P)] for x in range(P)]
     if have_values:
         outs = []
         for x in range(P):
@@ -488,14 +515,15 @@ def simulate(P: int, n: int, steps: int, inputs=None, op: str = "sum",
     return run
 
 
-def allreduce(inputs, steps: int, op: str = "sum", dtype: str = "f32", elements=None):
+def allreduce(inputs, steps: int, op: str = "sum", dtype: str = "f32", elements=None,
+              group: str = "cyclic"):
     """MPI_Allreduce semantics (Sec. "Introduction"): every process ends with the
     op-reduction of all P input vectors.  Returns the list of P output arrays (over the
     selected elements when ``elements`` is given)."""
     P = len(inputs)
     n = len(inputs[0]) if P else 0
     return simulate(P, n, steps, inputs=inputs, op=op, dtype=dtype,
-                    elements=elements).outputs
+                    elements=elements, group=group).outputs
 
 
 # ---------------------------------------------------------------------------

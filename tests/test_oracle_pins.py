@@ -449,7 +449,7 @@ def test_pins_pass_unmodified():
 
 
 def test_planted_wrong_partner_is_caught(monkeypatch):
-    monkeypatch.setattr(G, "_reduce_partner", lambda x, d, P: (x + d) % P)
+    monkeypatch.setattr(G, "_reduce_partner", lambda x, d, P, group="cyclic": (x + d) % P)
     assert not _pins_pass()
 
 
@@ -467,3 +467,120 @@ def test_planted_floor_halving_is_caught(monkeypatch):
         return Ns
     monkeypatch.setattr(G, "vector_counts", bad_counts)
     assert not _pins_pass()
+
+
+# ---------------------------------------------------------------------------
+# The self-inverse group of Table 1b (XOR group, P a power of two)
+# ---------------------------------------------------------------------------
+
+POW2 = [2, 4, 8, 16, 32, 64]
+
+
+def _textbook_recursive_halving(xs):
+    """Reduce-scatter by recursive vector halving, then allgather by recursive doubling,
+    with the partner at distance P/2 first (each rank keeps the half of its blocks whose
+    index agrees with its own rank in the exchanged bit).  Written from the textbook
+    description, independently of the oracle's schedule simulation."""
+    P, n = len(xs), len(xs[0])
+    bounds = G.block_bounds(n, P)
+    buf = [x.copy() for x in xs]
+    resp = [list(range(P)) for _ in range(P)]
+    m = P // 2
+    while m >= 1:
+        new = [b.copy() for b in buf]
+        new_resp = []
+        for x in range(P):
+            y = x ^ m
+            keep = [b for b in resp[x] if (b & m) == (x & m)]
+            for b in keep:
+                lo, hi = bounds[b]
+                new[x][lo:hi] = buf[x][lo:hi] + buf[y][lo:hi]
+            new_resp.append(keep)
+        buf, resp = new, new_resp
+        m //= 2
+    m = 1
+    while m < P:
+        new = [b.copy() for b in buf]
+        new_resp = []
+        for x in range(P):
+            y = x ^ m
+            for b in resp[y]:
+                lo, hi = bounds[b]
+                new[x][lo:hi] = buf[y][lo:hi]
+            new_resp.append(resp[x] + resp[y])
+        buf, resp = new, new_resp
+        m *= 2
+    return buf
+
+
+def _textbook_recursive_doubling(xs):
+    """Every rank exchanges its whole vector with the partner at distance P/2, P/4, ...,
+    1 and adds the partner's vector to its own."""
+    P = len(xs)
+    v = [x.copy() for x in xs]
+    m = P // 2
+    while m >= 1:
+        v = [v[x] + v[x ^ m] for x in range(P)]
+        m //= 2
+    return v
+
+
+@pytest.mark.parametrize("P", POW2)
+def test_xor_group_bo_is_recursive_halving(P):
+    """Sec. "Bandwidth-optimal algorithm": with P a power of two and the group of Table
+    1b the bandwidth-optimal algorithm is Recursive Halving -- same bits in float32."""
+    rng = np.random.default_rng(P)
+    n = 5 * P + 3
+    xs = [(rng.standard_normal(n) * np.exp2(rng.integers(-20, 21, n))).astype(np.float32)
+          for _ in range(P)]
+    L = G.ceil_log2(P)
+    got = G.allreduce(xs, 2 * L, "sum", "f32", group="xor")
+    want = _textbook_recursive_halving(xs)
+    for x in range(P):
+        np.testing.assert_array_equal(got[x].view(np.uint32), want[x].view(np.uint32))
+
+
+@pytest.mark.parametrize("P", POW2)
+def test_xor_group_lo_is_recursive_doubling(P):
+    """Sec. "Moving towards latency-optimal version": with the group of Table 1b the
+    latency-optimal algorithm is Recursive Doubling -- same bits in float32."""
+    rng = np.random.default_rng(100 + P)
+    n = 3 * P + 1
+    xs = [(rng.standard_normal(n) * np.exp2(rng.integers(-20, 21, n))).astype(np.float32)
+          for _ in range(P)]
+    got = G.allreduce(xs, G.ceil_log2(P), "sum", "f32", group="xor")
+    want = _textbook_recursive_doubling(xs)
+    for x in range(P):
+        np.testing.assert_array_equal(got[x].view(np.uint32), want[x].view(np.uint32))
+
+
+@pytest.mark.parametrize("P", POW2)
+def test_xor_group_coverage_bruteforce_and_traffic(P):
+    """Every result covers every rank once, int32 results are the column sums, and the
+    per-rank traffic is Recursive Halving's 2(P-1) blocks (S = 2L), Recursive Doubling's
+    P L blocks (S = L), and 2(P - K) + r K blocks in between (K = 2^r result copies: r
+    halving steps are replaced by doubling steps on K-block vectors)."""
+    L = G.ceil_log2(P)
+    rng = np.random.default_rng(7 * P)
+    n = 2 * P + 1
+    xs = [rng.integers(-1000, 1001, n).astype(np.int32) for _ in range(P)]
+    ref = G.column_reduce_exact(xs, "sum", "i32")
+    for S in range(L, 2 * L + 1):
+        run = G.simulate(P, n, S, inputs=xs, dtype="i32", group="xor")
+        for o in run.outputs:
+            np.testing.assert_array_equal(o, ref)
+        for key in set(k for row in run.out_key for k in row):
+            assert sorted(run.exprs.leaves(key[1])) == list(range(P))
+        r, K = run.r, run.K
+        assert K == 2 ** r
+        for x in range(P):
+            assert run.message_blocks_per_rank(x) == 2 * (P - K) + r * K
+        for st in run.log:
+            d = st["d"]
+            for (src, dst, _items) in st["messages"]:
+                assert dst == src ^ d          # pairwise exchange partners
+
+
+def test_xor_group_needs_power_of_two():
+    with pytest.raises(ValueError):
+        G.simulate(6, 0, 4, group="xor")
