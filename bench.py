@@ -509,8 +509,33 @@ def measure_rows(gar, gar_inputs, stream, hbm_peak):
             "GB/s": round(nbytes / ms / 1e6, 1), "frac": round(nbytes / ms / 1e6 / hbm_peak, 4)}
     del flat, out
     torch.cuda.empty_cache()
+    rows["groups_p64_4mib_f32"] = groups_row(gar, gar_inputs, stream, hbm_peak)
     rows["cost_model_p127_bf16_step"] = cost_model_row(gar, gar_inputs, stream)
     return rows
+
+
+def groups_row(gar, gar_inputs, stream, hbm_peak, P=64, n=1 << 20):
+    """Cyclic group (Table 1a) against the XOR group (Table 1b: Recursive Halving at
+    S = 2L, Recursive Doubling at S = L, their hybrid in between) for P = 64 x 4 MiB
+    fp32: per-rank message volume and step-faithful / fused times."""
+    import torch
+    inp = gar_inputs.rank_inputs(P, n, "f32", ("normal", 0.0, 1.0), 11, device="cuda")
+    L = _l(P)
+    out = {}
+    for group in ("cyclic", "xor"):
+        for S in (L, L + 2, 2 * L - 1, 2 * L):
+            plan = gar.gar_plan_create_group(P, n, "f32", "sum", S, group)
+            gar.ensure_workspace(plan)
+            gar.gar_plan_prepare(plan, "step")
+            gar.gar_plan_prepare(plan, "fused")
+            ms_s = _time_loop(lambda: gar.gar_allreduce(plan, inp, "step", stream), 5, 2, stream)
+            ms_f = _time_loop(lambda: gar.gar_allreduce(plan, inp, "fused", stream), 10, 2, stream)
+            out[f"{group}_S{S}"] = {"msg_bytes_per_rank": sum(gar.gar_plan_bytes(plan)[1]) // P,
+                                    "step_ms": round(ms_s, 4), "fused_ms": round(ms_f, 4)}
+            plan.workspace = None
+            del plan
+            torch.cuda.empty_cache()
+    return out
 
 
 def _paper_blocks(P, S):

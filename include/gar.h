@@ -70,6 +70,13 @@ enum { GAR_SUM = 0, GAR_MAX = 1, GAR_MIN = 2 };
  *   GAR_STEP_FAITHFUL. */
 enum { GAR_STEP_FAITHFUL = 0, GAR_FUSED = 1, GAR_STEP_PERSISTENT = 2 };
 
+/* The permutation group T_P (Sec. "Communication description via permutations").
+ * GAR_GROUP_CYCLIC: t_k(x) = x + k mod P (Table 1a), any P.
+ * GAR_GROUP_XOR: t_k(x) = x XOR k, the self-inverse group of Table 1b, P a power of two;
+ *   the bandwidth-optimal schedule is then Recursive Halving and the latency-optimal one
+ *   Recursive Doubling (every step a pairwise exchange with rank x XOR N_i/2). */
+enum { GAR_GROUP_CYCLIC = 0, GAR_GROUP_XOR = 1 };
+
 /* Special values for the `steps` argument of gar_plan_create. */
 #define GAR_STEPS_BO (-1) /* 2 ceil(log2 P): bandwidth-optimal */
 #define GAR_STEPS_LO (-2) /* ceil(log2 P): latency-optimal */
@@ -106,6 +113,7 @@ typedef struct {
   int32_t fused_width;       /* elements per thread-vector in the fused kernel (0 until compiled) */
   int32_t fused_regs;        /* registers per thread of the loaded fused kernel (0 until loaded) */
   int32_t fused_local_bytes; /* local (spill) bytes per thread of the loaded fused kernel */
+  int32_t group;             /* GAR_GROUP_CYCLIC or GAR_GROUP_XOR */
 } gar_plan_info;
 
 /* Creates a schedule for P virtual ranks of n elements each.
@@ -115,6 +123,13 @@ typedef struct {
  * initial_data) with the first n mod P blocks one element longer.  Host-only: needs
  * no GPU.  *out is set only on success. */
 GAR_API int gar_plan_create(gar_plan **out, int P, uint64_t n, int dtype, int op, int steps);
+
+/* gar_plan_create with an explicit group T_P (GAR_GROUP_*); gar_plan_create uses the
+ * cyclic group.  GAR_GROUP_XOR with P not a power of two returns GAR_EINVAL.  With the
+ * XOR group, K = 2^r result copies (r = 2L - S): the intermediate step counts are the
+ * Recursive Halving / Recursive Doubling hybrid. */
+GAR_API int gar_plan_create_group(gar_plan **out, int P, uint64_t n, int dtype, int op, int steps,
+                                  int group);
 
 /* Frees the plan and its device tables.  NULL is a no-op.  The caller must make sure
  * no work using the plan is still running. */
@@ -253,7 +268,7 @@ GAR_API int gar_cost_model(int P, int steps, double m_bytes, double alpha, doubl
 GAR_API int gar_optimal_steps(int P, double m_bytes, double alpha, double beta, double gamma,
                               int *steps);
 
-/* Step-faithful Allreduce that allocates no device memory.  The paper has no
+/* Step-faithful Allreduce that allocates no device memory (cyclic-group plans only).  The paper has no
  * counterpart; this entry point serves callers that cannot call cudaMalloc when they
  * run an Allreduce, e.g. code whose device memory is all owned by a caching
  * allocator or by another runtime.  Same result as gar_allreduce(plan, rank_buffers,

@@ -298,6 +298,10 @@ using namespace gar;
 extern "C" {
 
 int gar_plan_create(gar_plan **out, int P, uint64_t n, int dtype, int op, int steps) {
+  return gar_plan_create_group(out, P, n, dtype, op, steps, GAR_GROUP_CYCLIC);
+}
+
+int gar_plan_create_group(gar_plan **out, int P, uint64_t n, int dtype, int op, int steps, int group) {
   if (out == nullptr) {
     set_error("null output pointer");
     return GAR_EINVAL;
@@ -318,6 +322,14 @@ int gar_plan_create(gar_plan **out, int P, uint64_t n, int dtype, int op, int st
     set_error("n too large");
     return GAR_EINVAL;
   }
+  if (group != GAR_GROUP_CYCLIC && group != GAR_GROUP_XOR) {
+    set_error("unknown group");
+    return GAR_EINVAL;
+  }
+  if (group == GAR_GROUP_XOR && (P & (P - 1)) != 0) {
+    set_error("the XOR group needs P a power of two");
+    return GAR_EINVAL;
+  }
   const int L = ceil_log2(P);
   int S = steps;
   if (steps == GAR_STEPS_BO) S = 2 * L;
@@ -334,6 +346,7 @@ int gar_plan_create(gar_plan **out, int P, uint64_t n, int dtype, int op, int st
   pl->dtype = dtype;
   pl->op = op;
   pl->S = S;
+  pl->group = group;
   int rc = build_plan(pl);
   if (rc) {
     delete pl;
@@ -375,6 +388,7 @@ int gar_plan_get_info(const gar_plan *pl, gar_plan_info *info) {
   info->n_launches = (int)pl->launches.size();
   info->n = pl->n;
   info->fused_combines = (int)pl->prog.a.size();
+  info->group = pl->group;
   info->fused_width = pl->fused_width;
   if (pl->fused != nullptr && pl->fused->loaded) {
     info->fused_regs = pl->fused->regs;

@@ -255,15 +255,17 @@ std::string emit_eval(const FusedProgram &fp, const Schedule &sc, const std::str
                       const std::string &params,
                       const std::function<std::string(const std::string &)> &ld_row,
                       const std::function<std::string(const std::string &)> &st_row,
-                      bool rotate) {
+                      bool rotate, bool xor_group) {
   const int P = fp.P;
   std::string s;
   s += "template <int W>\nstatic __device__ __forceinline__ void gar_eval_" + tag + "(" + params +
        ", gar_u64 e0, int b) {\n";
   s += "  (void)b;\n";
+  // rank of contribution / placement j for an element of block b: t_j(b)
   auto rank_of = [&](int j) -> std::string {
     if (!rotate) return std::to_string(j);
     if (j == 0) return "b";
+    if (xor_group) return fmt("(b ^ %d)", j);
     return fmt("(b + %d >= %d ? b + %d : b + %d)", j, P, j - P, j);
   };
   // stores of result s go to every placement p whose origin is s
@@ -325,7 +327,7 @@ CodegenResult generate_fused_source(const gar_plan &pl) {
   CodegenResult cg;
   cg.width = W;
   cg.kernel_name = fmt("gar_fused_P%d_S%d_K%d_", P, pl.S, pl.K) + dtype_tag(pl.dtype) + "_" +
-                   op_tag(pl.op) + fmt("_W%d", W);
+                   op_tag(pl.op) + fmt("_W%d", W) + (pl.group == GAR_GROUP_XOR ? "_xor" : "");
   std::string s;
   s += fmt("#define GAR_DTYPE %d\n#define GAR_OP %d\n", pl.dtype, pl.op);
   s += "#define GAR_LDH \"" + tune_str("GAR_TUNE_LDH", ".cs") + "\"\n";
@@ -340,7 +342,8 @@ CodegenResult generate_fused_source(const gar_plan &pl) {
   s += emit_block_of("gar_block_of", P, pl.n);
   auto ld_row = [](const std::string &r) { return "a.in[" + r + "]"; };
   auto st_row = [](const std::string &r) { return "a.out[" + r + "]"; };
-  s += emit_eval(fp, sc, "plan", "const gar_args &a", ld_row, st_row, rotate);
+  s += emit_eval(fp, sc, "plan", "const gar_args &a", ld_row, st_row, rotate,
+                 pl.group == GAR_GROUP_XOR);
   s += "extern \"C\" __global__ void " + bounds + " " + cg.kernel_name +
        "(const __grid_constant__ gar_args a) {\n";
   s += "  const gar_u64 v_lo = a.e_lo / GAR_W, v_hi = a.e_hi / GAR_W;\n";
@@ -382,7 +385,8 @@ CodegenResult generate_batched_source(const std::vector<const gar_plan *> &plans
   CodegenResult cg;
   cg.width = W;
   std::string name = "gar_batched_";
-  for (const gar_plan *pl : plans) name += fmt("P%dS%d_", pl->P, pl->S);
+  for (const gar_plan *pl : plans)
+    name += fmt("P%dS%d", pl->P, pl->S) + (pl->group == GAR_GROUP_XOR ? "x_" : "_");
   cg.kernel_name = name + dtype_tag(p0.dtype) + "_" + op_tag(p0.op) + fmt("_W%d", W);
   std::string s;
   s += fmt("#define GAR_DTYPE %d\n#define GAR_OP %d\n", p0.dtype, p0.op);
@@ -401,7 +405,8 @@ CodegenResult generate_batched_source(const std::vector<const gar_plan *> &plans
     s += emit_block_of("gar_block_of_" + tag, pl.P, pl.n);
     auto ld = [](const std::string &r) { return "(in + GAR_N * (gar_u64)(" + r + "))"; };
     auto st = [](const std::string &r) { return "(out + GAR_N * (gar_u64)(" + r + "))"; };
-    s += emit_eval(pl.prog, scs[k], tag, "const gar_io *in, gar_io *out", ld, st, rotate);
+    s += emit_eval(pl.prog, scs[k], tag, "const gar_io *in, gar_io *out", ld, st, rotate,
+                   pl.group == GAR_GROUP_XOR);
   }
   s += "extern \"C\" __global__ void __launch_bounds__(256) " + cg.kernel_name +
        "(const __grid_constant__ gar_bargs a) {\n";

@@ -53,7 +53,7 @@ struct CommStep {
   int phase;                      // 0 reduce, 1 distribute
   int i;                          // the paper's step index i
   int N, d;
-  int partner;
+  int partner;                    // cyclic: rank x receives from x + partner; XOR: x ^ partner
   std::vector<int32_t> tx;        // placements transmitted by every rank
   uint64_t msg_bytes;             // predicted, all ranks together
 };
@@ -74,6 +74,7 @@ constexpr int GAR_HOST_CHUNKS_MAX = 16;  // element chunks of the pipelined host
 
 struct gar_plan {
   int P = 0, L = 0, S = 0, r = 0, K = 0;
+  int group = 0;                  // GAR_GROUP_CYCLIC or GAR_GROUP_XOR
   uint64_t n = 0;
   int dtype = 0, op = 0;
   uint64_t q = 0, rem = 0;        // block i has q + (i < rem) elements

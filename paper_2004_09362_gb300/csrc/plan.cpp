@@ -20,6 +20,10 @@
 //    extra vector t^{N_i} q'_{N_i} per added copy, Sec. "Moving towards latency-optimal
 //    version"), and each received vector is combined into the q' and/or q* at its new
 //    placement.
+// With the self-inverse group of Table 1b (P a power of two) every "+" on placements and
+// ranks becomes XOR: placement p puts block i on rank i ^ p, the step operator is
+// t_{N_i/2} (x -> x ^ N_i/2), copy s has index k at placement s ^ k, and the unions of
+// the copies' placement sets are enumerated instead of taken as ranges.
 #include <algorithm>
 #include <map>
 #include <stdexcept>
@@ -52,6 +56,32 @@ std::vector<int32_t> placement_range(long lo, long hi, int P) {
       out.push_back(p);
     }
   }
+  return out;
+}
+
+// Group operation t_a(b) and inverse on {0..P-1}: cyclic (Table 1a) or XOR (Table 1b).
+struct Group {
+  int P;
+  bool xr;
+  int op(int a, int b) const { return xr ? (a ^ b) : (a + b) % P; }
+  int inv(int a) const { return xr ? a : (P - a) % P; }
+};
+
+// Placements t_s(k) for s in [0, K), k in [lo, hi], each once.  Cyclic: the
+// consecutive range [lo, K - 1 + hi] mod P (placement_range); XOR: enumerated.
+std::vector<int32_t> union_placements(const Group &g, int K, long lo, long hi) {
+  if (!g.xr) return placement_range(lo, (long)K - 1 + hi, g.P);
+  std::vector<int32_t> out;
+  if (hi < lo) return out;
+  std::vector<char> seen(g.P, 0);
+  for (int s = 0; s < K; ++s)
+    for (long k = lo; k <= hi; ++k) {
+      const int p = g.op(s, (int)k);
+      if (!seen[p]) {
+        seen[p] = 1;
+        out.push_back(p);
+      }
+    }
   return out;
 }
 
@@ -90,6 +120,7 @@ void add_out(StepOp &op, Buf dst, Buf own) {
 // and receivers [ceil(N/2), N-1] are disjoint placements).
 void build_step_faithful(gar_plan *pl) {
   const int P = pl->P, L = pl->L, K = pl->K, r = pl->r;
+  const Group g{P, pl->group == GAR_GROUP_XOR};
   const bool acc_is_elem = pl->dtype != GAR_BF16;
   const Buf inplace = acc_is_elem ? BUF_RANK : BUF_QP0;
   const Buf qs_loc = (K == 1) ? inplace : BUF_QS;
@@ -111,22 +142,22 @@ void build_step_faithful(gar_plan *pl) {
     }
     std::vector<char> in_next(P, 0);  // q' placements alive after this step
     if (c >= 2)
-      for (int32_t p : placement_range(1, (long)K + c - 2, P)) in_next[p] = 1;
+      for (int32_t p : union_placements(g, K, 1, c - 1)) in_next[p] = 1;
 
     CommStep cs;
     cs.phase = 0;
     cs.i = i;
     cs.N = N;
     cs.d = d;
-    cs.partner = d;
-    cs.tx = placement_range(c, (long)K + N - 2, P);
+    cs.partner = d;  // receive from the rank the step operator t_d^{-1} maps onto x
+    cs.tx = union_placements(g, K, c, N - 1);
     Launch ln;
     ln.phase = 0;
     ln.comm_step = (int)pl->comm.size();
     ln.partner = d;
     ln.first_op = (int)pl->ops.size();
     for (int32_t p : cs.tx) {
-      const int pp = ((p - d) % P + P) % P;  // placement after the move by t^{-d}
+      const int pp = g.op(p, g.inv(d));  // placement after the move by t_d^{-1}
       const bool to_qp = in_next[pp] != 0;
       const bool to_qs = even && pp < K;
       StepOp op = make_op(p, pp, src);
@@ -185,15 +216,15 @@ void build_step_faithful(gar_plan *pl) {
     cs.i = i;
     cs.N = N;
     cs.d = d;
-    cs.partner = -d;
+    cs.partner = g.xr ? d : -d;  // receive from t_d^{-1}(x): x - d, or x XOR d
     Launch ln;
     ln.phase = 1;
     ln.comm_step = (int)pl->comm.size();
-    ln.partner = -d;
+    ln.partner = cs.partner;
     ln.first_op = (int)pl->ops.size();
     for (int p = N % 2; p < c; ++p) {
       cs.tx.push_back(p);
-      StepOp op = make_op(p, (p + d) % P, BUF_RANK);
+      StepOp op = make_op(p, g.op(p, d), BUF_RANK);
       add_out(op, BUF_RANK, BUF_NONE);
       pl->ops.push_back(op);
     }
@@ -215,6 +246,7 @@ void build_step_faithful(gar_plan *pl) {
 // one value (the union of the shifted copies computes every distinct vector once).
 void build_fused(gar_plan *pl) {
   const int P = pl->P, L = pl->L, K = pl->K, r = pl->r;
+  const Group g{P, pl->group == GAR_GROUP_XOR};
   FusedProgram &fp = pl->prog;
   fp = FusedProgram{};
   fp.P = P;
@@ -240,9 +272,10 @@ void build_fused(gar_plan *pl) {
     const bool even = (N % 2 == 0);
     std::vector<int> nqp(P, -1), nqs(K);
     // q*_s first, then q'_p: the values are CSE'd, the order only fixes numbering
-    for (int s = 0; s < K; ++s) nqs[s] = even ? mk(qs[s], qp[(s + d) % P]) : qs[s];
+    // the vector received at placement p came from placement t_d(p)
+    for (int s = 0; s < K; ++s) nqs[s] = even ? mk(qs[s], qp[g.op(s, d)]) : qs[s];
     if (c >= 2)
-      for (int32_t p : placement_range(1, (long)K + c - 2, P)) nqp[p] = mk(qp[p], qp[(p + d) % P]);
+      for (int32_t p : union_placements(g, K, 1, c - 1)) nqp[p] = mk(qp[p], qp[g.op(p, d)]);
     qp.swap(nqp);
     qs.swap(nqs);
   }
@@ -275,7 +308,7 @@ void build_fused(gar_plan *pl) {
   for (int s = 0; s < K; ++s) fp.origin[s] = s;
   for (int i = L - r - 1; i >= 0; --i) {
     const int N = pl->N[i], d = N / 2, c = N - d;
-    for (int p = c; p < N; ++p) fp.origin[p] = fp.origin[p - d];
+    for (int p = N % 2; p < c; ++p) fp.origin[g.op(p, d)] = fp.origin[p];
   }
   for (int p = 0; p < P; ++p)
     if (fp.origin[p] < 0) throw std::logic_error("placement without a result");

@@ -46,6 +46,7 @@ struct StepArgs {
   uint64_t chunk;                    // elements per CTA
   uint64_t n;                        // elements per rank
   int P, partner, nops, nchunks;
+  int xor_group;                     // 1: placements and partners combine by XOR (Table 1b)
 };
 
 template <typename T> struct AccOf { using type = T; };
@@ -150,7 +151,7 @@ __device__ __forceinline__ void chunk_work(const StepArgs<MAXP> &a, const Launch
   const int oi = (int)(item / (uint64_t)a.P);
   if (oi >= lv.nops) return;
   const StepOp op = lv.ops[oi];
-  const int b = ((x - (int)op.dst_place) % a.P + a.P) % a.P;
+  const int b = a.xor_group ? (x ^ (int)op.dst_place) : ((x - (int)op.dst_place) % a.P + a.P) % a.P;
   const uint64_t bstart = (uint64_t)b * a.q + ((uint64_t)b < a.rem ? (uint64_t)b : a.rem);
   const uint64_t blen = a.q + ((uint64_t)b < a.rem ? 1 : 0);
   const uint64_t c0 = (uint64_t)chunk * lv.chunk;
@@ -159,7 +160,7 @@ __device__ __forceinline__ void chunk_work(const StepArgs<MAXP> &a, const Launch
   const uint64_t hi = bstart + (blen < c0 + lv.chunk ? blen : c0 + lv.chunk);
 
   const bool has_recv = op.recv_place >= 0;
-  const int partner = ((x + lv.partner) % a.P + a.P) % a.P;
+  const int partner = a.xor_group ? (x ^ lv.partner) : ((x + lv.partner) % a.P + a.P) % a.P;
   const void *recv = has_recv ? buf_ptr<A>(a, op.recv_buf, partner) : nullptr;
   void *out0 = buf_ptr<A>(a, op.out0_buf, x);
   const void *own0 = buf_ptr<A>(a, op.out0_own, x);
@@ -250,11 +251,11 @@ __device__ __forceinline__ void flat_work(const StepArgs<MAXP> &a, const LaunchV
     const uint64_t e = g - (uint64_t)oi * a.n;
     const StepOp op = lv.ops[oi];
     const int b = e < big ? (int)(e / (a.q + 1)) : (int)(a.rem + (e - big) / a.q);
-    const int x = (b + (int)op.dst_place) % a.P;
+    const int x = a.xor_group ? (b ^ (int)op.dst_place) : (b + (int)op.dst_place) % a.P;
     A r = A(0);
     const bool has_recv = op.recv_place >= 0;
     if (has_recv) {
-      const int partner = ((x + lv.partner) % a.P + a.P) % a.P;
+      const int partner = a.xor_group ? (x ^ lv.partner) : ((x + lv.partner) % a.P + a.P) % a.P;
       r = load1<T, A>(op.recv_buf, buf_ptr<A>(a, op.recv_buf, partner), e);
       moved_bytes += (op.recv_buf == BUF_RANK) ? sizeof(T) : sizeof(A);
     }
@@ -433,6 +434,7 @@ int launch_typed(const gar_plan &pl, const Launch &ln, int launch_index, void *c
   a.n_pad = pl.n_pad;
   a.n = pl.n;
   a.P = pl.P;
+  a.xor_group = pl.group == GAR_GROUP_XOR ? 1 : 0;
   a.partner = ln.partner;
   a.nops = ln.nops;
   const uint64_t maxblk = pl.q + (pl.rem ? 1 : 0);
@@ -497,6 +499,7 @@ int launch_persistent_typed(const gar_plan &pl, void *const *rank, gar_stream_t 
   p.s.n_pad = pl.n_pad;
   p.s.n = pl.n;
   p.s.P = pl.P;
+  p.s.xor_group = pl.group == GAR_GROUP_XOR ? 1 : 0;
   const uint64_t maxblk = pl.q + (pl.rem ? 1 : 0);
   p.flat = maxblk < kFlatBelow ? 1 : 0;
   p.s.chunk = kChunk;
@@ -735,6 +738,10 @@ extern "C" int gar_allreduce_noalloc(gar_plan *pl, void *const *rank_buffers, ga
   using namespace gar;
   if (pl == nullptr || rank_buffers == nullptr) {
     set_error("null plan or rank buffer array");
+    return GAR_EINVAL;
+  }
+  if (pl->group != GAR_GROUP_CYCLIC) {
+    set_error("gar_allreduce_noalloc supports the cyclic group only");
     return GAR_EINVAL;
   }
   if (pl->P > GAR_NOALLOC_MAX_P) {

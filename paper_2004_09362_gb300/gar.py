@@ -20,6 +20,8 @@ GAR_F32, GAR_BF16, GAR_I32 = 0, 1, 2
 GAR_SUM, GAR_MAX, GAR_MIN = 0, 1, 2
 GAR_STEP_FAITHFUL, GAR_FUSED, GAR_STEP_PERSISTENT = 0, 1, 2
 GAR_STEPS_BO, GAR_STEPS_LO = -1, -2
+GAR_GROUP_CYCLIC, GAR_GROUP_XOR = 0, 1
+GROUPS = {"cyclic": GAR_GROUP_CYCLIC, "xor": GAR_GROUP_XOR}
 GAR_MAX_P = 1024
 GAR_OK = 0
 
@@ -37,6 +39,7 @@ EXPORTS = (
     "gar_allreduce_host", "gar_allreduce_batched", "gar_last_step_bytes", "gar_strerror",
     "gar_last_error", "gar_selftest_compile", "gar_allreduce_noalloc", "gar_plan_fused_source",
     "gar_cost_model", "gar_optimal_steps", "gar_plan_status", "gar_plan_debug_barrier",
+    "gar_plan_create_group",
 )
 
 
@@ -51,7 +54,8 @@ class gar_plan_info(ctypes.Structure):
                 ("r", ctypes.c_int32), ("K", ctypes.c_int32), ("dtype", ctypes.c_int32),
                 ("op", ctypes.c_int32), ("n_launches", ctypes.c_int32), ("n", ctypes.c_uint64),
                 ("fused_combines", ctypes.c_int32), ("fused_width", ctypes.c_int32),
-                ("fused_regs", ctypes.c_int32), ("fused_local_bytes", ctypes.c_int32)]
+                ("fused_regs", ctypes.c_int32), ("fused_local_bytes", ctypes.c_int32),
+                ("group", ctypes.c_int32)]
 
 
 def _load():
@@ -62,6 +66,7 @@ def _load():
     P_ = ctypes.POINTER
     sig = {
         "gar_plan_create": (i32, [P_(vp), i32, u64, i32, i32, i32]),
+        "gar_plan_create_group": (i32, [P_(vp), i32, u64, i32, i32, i32, i32]),
         "gar_plan_destroy": (None, [vp]),
         "gar_plan_get_info": (i32, [vp, P_(gar_plan_info)]),
         "gar_plan_bytes": (i32, [vp, P_(sz), P_(u64), P_(i32)]),
@@ -156,6 +161,15 @@ def gar_plan_create(P: int, n: int, dtype="f32", op="sum", steps=GAR_STEPS_BO) -
     h = ctypes.c_void_p()
     _check(_lib.gar_plan_create(ctypes.byref(h), int(P), int(n), _code(dtype, DTYPES, "dtype"),
                                 _code(op, OPS, "op"), int(steps)), "gar_plan_create")
+    return Plan(h.value)
+
+
+def gar_plan_create_group(P: int, n: int, dtype="f32", op="sum", steps=GAR_STEPS_BO,
+                          group="cyclic") -> Plan:
+    h = ctypes.c_void_p()
+    _check(_lib.gar_plan_create_group(ctypes.byref(h), int(P), int(n), _code(dtype, DTYPES, "dtype"),
+                                      _code(op, OPS, "op"), int(steps), _code(group, GROUPS, "group")),
+           "gar_plan_create_group")
     return Plan(h.value)
 
 

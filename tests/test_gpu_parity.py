@@ -346,6 +346,57 @@ def test_batched_mixed_order_and_steps():
 
 
 # ---------------------------------------------------------------------------
+# The XOR group (Table 1b): Recursive Halving / Doubling and their hybrids
+# ---------------------------------------------------------------------------
+
+def _run_group(P, n, dtype, S, mode, t, group):
+    plan = gar.gar_plan_create_group(P, n, dtype, "sum", S, group)
+    return plan, _run(plan, t, mode)
+
+
+@pytest.mark.parametrize("P", [2, 4, 8, 16, 32, 64])
+@pytest.mark.parametrize("mode", ["fused", "step", "persistent"])
+def test_xor_group_matches_oracle(P, mode):
+    cases = [(2 * P + 3, "f32"), (2 * P + 3, "i32"), (2 * P + 3, "bf16"), (P * 4099 + 1, "f32")]
+    for (n, dtype) in cases:
+        t = _np_inputs(P, n, dtype, seed=17 * P + n)
+        host = _to_host_list(t, dtype)
+        for S in _Ss(P):
+            plan, got = _run_group(P, n, dtype, S, mode, t, "xor")
+            _assert_same(got, G.allreduce(host, S, "sum", dtype, group="xor"), dtype,
+                         f"xor P={P} n={n} {dtype} S={S} {mode}")
+            if mode != "fused":
+                assert gar.gar_last_step_bytes(plan) == gar.gar_plan_bytes(plan)[1]
+
+
+def test_batched_mixed_groups():
+    n = 64
+    plans = [gar.gar_plan_create_group(8, n, "f32", "sum", 4, "xor"),
+             gar.gar_plan_create_group(6, n, "f32", "sum", 4, "cyclic"),
+             gar.gar_plan_create_group(16, n, "f32", "sum", 4, "xor")]
+    Ps, steps, groups = (8, 6, 16), (4, 4, 4), ("xor", "cyclic", "xor")
+    count = 90
+    which = [i % 3 for i in range(count)]
+    sizes = [Ps[w] * n for w in which]
+    offs = np.concatenate([[0], np.cumsum(sizes)])[:-1]
+    data = torch.randn(int(offs[-1] + sizes[-1]), device=DEV)
+    ref_in = data.cpu().numpy().copy()
+    desc = gar.make_batch_desc(which, [data.data_ptr() + int(o) * 4 for o in offs],
+                               [data.data_ptr() + int(o) * 4 for o in offs])
+    gar.gar_allreduce_batched(plans, desc, count)
+    torch.cuda.synchronize()
+    got = data.cpu().numpy()
+    for i in range(count):
+        w, o = which[i], int(offs[i])
+        P = Ps[w]
+        xs = [ref_in[o + x * n: o + (x + 1) * n].copy() for x in range(P)]
+        want = G.allreduce(xs, steps[w], "sum", "f32", group=groups[w])
+        for x in range(P):
+            np.testing.assert_array_equal(got[o + x * n: o + (x + 1) * n].view(np.uint32),
+                                          want[x].view(np.uint32))
+
+
+# ---------------------------------------------------------------------------
 # Persistent step-faithful mode: one cooperative launch, bounded grid barriers
 # ---------------------------------------------------------------------------
 

@@ -45,17 +45,22 @@ def _cases():
     for P in list(range(1, 41)) + [63, 64, 65, 127, 128, 129]:
         L = G.ceil_log2(P)
         for S in range(L, 2 * L + 1):
-            out.append((P, S))
+            out.append((P, S, "cyclic"))
+    for P in (1, 2, 4, 8, 16, 32, 64, 128):
+        L = G.ceil_log2(P)
+        for S in range(L, 2 * L + 1):
+            out.append((P, S, "xor"))
     return out
 
 
-@pytest.mark.parametrize("P,S", _cases())
-def test_schedule_matches_oracle(P, S):
+@pytest.mark.parametrize("P,S,group", _cases())
+def test_schedule_matches_oracle(P, S, group):
     n = 3 * P + 1 if P > 1 else 5
     for dtype in ("f32", "bf16"):
-        plan = gar.gar_plan_create(P, n, dtype, "sum", S)
+        plan = gar.gar_plan_create_group(P, n, dtype, "sum", S, group)
         info = plan.info()
-        run = G.simulate(P, n, S, dtype=dtype)
+        assert info["group"] == gar.GROUPS[group]
+        run = G.simulate(P, n, S, dtype=dtype, group=group)
         assert (info["L"], info["S"], info["r"], info["K"]) == (run.L, run.steps, run.r, run.K)
         ws, per_step, S_lib = gar.gar_plan_bytes(plan)
         assert S_lib == S
@@ -63,7 +68,10 @@ def test_schedule_matches_oracle(P, S):
         for t, st in enumerate(run.log):
             phase, partner, tx = gar.gar_plan_step(plan, t)
             assert phase == (0 if st["phase"] == "reduce" else 1)
-            assert partner == (st["d"] if phase == 0 else -st["d"])
+            if group == "xor":
+                assert partner == st["d"]
+            else:
+                assert partner == (st["d"] if phase == 0 else -st["d"])
             assert sorted(tx) == sorted(k[0] for k in st["tx"])
         # origin map: rank x's block b comes from placement (x - b); its tree is copy o
         origin = gar.gar_plan_origin(plan)
@@ -109,7 +117,7 @@ def _op(op, a, b):
     return np.maximum(a, b) if op == "max" else np.minimum(a, b)
 
 
-def emulate_step_faithful(plan, xs, dtype, op):
+def emulate_step_faithful(plan, xs, dtype, op, group="cyclic"):
     """Executes the plan's step-faithful op table on the CPU.  Rank buffers hold the
     element type (bf16 values kept as float32 after rounding), workspace the
     accumulation type.  Returns (outputs, per-launch recv element counts)."""
@@ -122,17 +130,19 @@ def emulate_step_faithful(plan, xs, dtype, op):
             BUF_QP1: [np.zeros(n, acc_dt) for _ in range(P)],
             BUF_QS: [np.zeros(n, acc_dt) for _ in range(P)]}
     ops, partners = gar.gar_plan_step_ops(plan)
+    xr = group == "xor"
     for l, partner in enumerate(partners):
         lops = ops[ops[:, 0] == l]
         writes, reads, written = [], set(), {}
         for (_l, recv_place, dst_place, recv_buf, o0b, o0o, o1b, o1o) in lops:
             for x in range(P):
-                b = (x - dst_place) % P
+                b = (x ^ dst_place) if xr else (x - dst_place) % P
                 lo, hi = bounds[b]
                 recv = None
                 if recv_place >= 0:
-                    src = (x + partner) % P
-                    assert (src - recv_place) % P == b      # same block at the partner
+                    src = (x ^ partner) if xr else (x + partner) % P
+                    # the partner holds the same block at the transmitted placement
+                    assert ((src ^ recv_place) if xr else (src - recv_place) % P) == b
                     recv = _to_acc(bufs[recv_buf][src][lo:hi], dtype)
                     reads.add((recv_buf, src, b))
                 for (ob, oo) in ((o0b, o0o), (o1b, o1o)):
@@ -158,8 +168,9 @@ def emulate_step_faithful(plan, xs, dtype, op):
     return bufs[BUF_RANK]
 
 
-@pytest.mark.parametrize("P", list(range(1, 18)) + [24, 31, 33])
-def test_step_faithful_tables_reproduce_oracle(P):
+@pytest.mark.parametrize("P,group", [(P, "cyclic") for P in list(range(1, 18)) + [24, 31, 33]]
+                         + [(P, "xor") for P in (1, 2, 4, 8, 16, 32)])
+def test_step_faithful_tables_reproduce_oracle(P, group):
     rng = np.random.default_rng(P)
     L = G.ceil_log2(P)
     for n in sorted({max(P - 1, 1), 2 * P + 3}):
@@ -172,30 +183,32 @@ def test_step_faithful_tables_reproduce_oracle(P):
                 if dtype == "bf16":
                     xs = [G.round_to_bf16(v) for v in xs]
             for S in range(L, 2 * L + 1):
-                plan = gar.gar_plan_create(P, n, dtype, "sum", S)
-                got = emulate_step_faithful(plan, xs, dtype, "sum")
-                want = G.allreduce(xs, S, "sum", dtype)
+                plan = gar.gar_plan_create_group(P, n, dtype, "sum", S, group)
+                got = emulate_step_faithful(plan, xs, dtype, "sum", group)
+                want = G.allreduce(xs, S, "sum", dtype, group=group)
                 for x in range(P):
                     np.testing.assert_array_equal(got[x].view(np.uint32), want[x].view(np.uint32))
 
 
-def emulate_fused(plan, xs, op):
+def emulate_fused(plan, xs, op, group="cyclic"):
     P = len(xs)
     n = len(xs[0])
     pairs, outs = gar.gar_plan_fused_program(plan)
     origin = gar.gar_plan_origin(plan)
+    t = (lambda b, j: b ^ j) if group == "xor" else (lambda b, j: (b + j) % P)
     res = [np.empty_like(x) for x in xs]
     for b, (lo, hi) in enumerate(_blocks(n, P)):
-        vals = [xs[(b + j) % P][lo:hi] for j in range(P)]
+        vals = [xs[t(b, j)][lo:hi] for j in range(P)]
         for (a, c) in pairs:
             vals.append(_op(op, vals[a], vals[c]))
         for p in range(P):
-            res[(b + p) % P][lo:hi] = vals[outs[origin[p]]]
+            res[t(b, p)][lo:hi] = vals[outs[origin[p]]]
     return res
 
 
-@pytest.mark.parametrize("P", list(range(1, 20)) + [24, 40, 127])
-def test_fused_program_reproduces_oracle(P):
+@pytest.mark.parametrize("P,group", [(P, "cyclic") for P in list(range(1, 20)) + [24, 40, 127]]
+                         + [(P, "xor") for P in (2, 4, 8, 16, 64, 128)])
+def test_fused_program_reproduces_oracle(P, group):
     rng = np.random.default_rng(1000 + P)
     L = G.ceil_log2(P)
     n = 2 * P + 5
@@ -203,9 +216,9 @@ def test_fused_program_reproduces_oracle(P):
           for _ in range(P)]
     for S in range(L, 2 * L + 1):
         for op in ("sum", "max"):
-            plan = gar.gar_plan_create(P, n, "f32", op, S)
-            got = emulate_fused(plan, xs, op)
-            want = G.allreduce(xs, S, op, "f32")
+            plan = gar.gar_plan_create_group(P, n, "f32", op, S, group)
+            got = emulate_fused(plan, xs, op, group)
+            want = G.allreduce(xs, S, op, "f32", group=group)
             for x in range(P):
                 np.testing.assert_array_equal(got[x].view(np.uint32), want[x].view(np.uint32))
 
@@ -223,6 +236,13 @@ def test_workspace_sizes():
     assert ws == 2 * 8 * 1024 * 4          # P = 2^k: q* never separates from q'
     ws, _, _ = gar.gar_plan_bytes(gar.gar_plan_create(7, 1000, "f32", "sum", gar.GAR_STEPS_LO))
     assert ws == 3 * 7 * 1024 * 4
+
+
+def test_group_argument_errors():
+    with pytest.raises(gar.GarError):
+        gar.gar_plan_create_group(6, 10, steps=3, group="xor")     # not a power of two
+    with pytest.raises(gar.GarError):
+        gar.gar_plan_create_group(8, 10, steps=3, group=7)
 
 
 def test_argument_errors():
