@@ -510,8 +510,33 @@ def measure_rows(gar, gar_inputs, stream, hbm_peak):
     del flat, out
     torch.cuda.empty_cache()
     rows["groups_p64_4mib_f32"] = groups_row(gar, gar_inputs, stream, hbm_peak)
+    rows["ring_vs_bo_p24_64mib_f32"] = ring_row(gar, gar_inputs, stream, hbm_peak)
     rows["cost_model_p127_bf16_step"] = cost_model_row(gar, gar_inputs, stream)
     return rows
+
+
+def ring_row(gar, gar_inputs, stream, hbm_peak):
+    """The Ring (2(P-1) steps, the far end of the paper's step range) against the
+    bandwidth-optimal schedule (2L steps) on the headline workload, both modes."""
+    import torch
+    wl = gar_inputs.WORKLOADS[HEADLINE]
+    P, n = wl.P, wl.n
+    inp = gar_inputs.rank_inputs(P, n, "f32", wl.dist, wl.seed, device="cuda")
+    out = {}
+    for name, steps in (("ring", gar.GAR_STEPS_RING), ("bandwidth_optimal", gar.GAR_STEPS_BO)):
+        plan = gar.gar_plan_create(P, n, "f32", "sum", steps)
+        gar.gar_plan_prepare(plan, "step")
+        gar.gar_plan_prepare(plan, "fused")
+        ms_s = _time_loop(lambda: gar.gar_allreduce(plan, inp, "step", stream), 5, 2, stream)
+        ms_f = _time_loop(lambda: gar.gar_allreduce(plan, inp, "fused", stream), 10, 2, stream)
+        dram = _step_dram_bytes(gar, plan, P, n, "f32")
+        out[name] = {"S": plan.info()["S"], "step_ms": round(ms_s, 4),
+                     "step_frac_dram_model": round(dram / ms_s / 1e6 / hbm_peak, 4),
+                     "fused_ms": round(ms_f, 4),
+                     "msg_bytes_per_rank": sum(gar.gar_plan_bytes(plan)[1]) // P}
+    del inp
+    torch.cuda.empty_cache()
+    return out
 
 
 def groups_row(gar, gar_inputs, stream, hbm_peak, P=64, n=1 << 20):

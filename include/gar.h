@@ -80,6 +80,10 @@ enum { GAR_GROUP_CYCLIC = 0, GAR_GROUP_XOR = 1 };
 /* Special values for the `steps` argument of gar_plan_create. */
 #define GAR_STEPS_BO (-1) /* 2 ceil(log2 P): bandwidth-optimal */
 #define GAR_STEPS_LO (-2) /* ceil(log2 P): latency-optimal */
+/* The Ring: the straightforward algorithm of Sec. "Allreduce as permutation composition"
+ * with the cyclic group, every step moving by the generator t (x -> x + 1); 2(P-1) steps
+ * (eq. naive_cost), the far end of the paper's step range.  Cyclic group only. */
+#define GAR_STEPS_RING (-3)
 
 #define GAR_MAX_P 1024 /* largest supported number of virtual ranks */
 
@@ -114,11 +118,13 @@ typedef struct {
   int32_t fused_regs;        /* registers per thread of the loaded fused kernel (0 until loaded) */
   int32_t fused_local_bytes; /* local (spill) bytes per thread of the loaded fused kernel */
   int32_t group;             /* GAR_GROUP_CYCLIC or GAR_GROUP_XOR */
+  int32_t ring;              /* 1 for the Ring schedule (GAR_STEPS_RING) */
 } gar_plan_info;
 
 /* Creates a schedule for P virtual ranks of n elements each.
  * P: 1..GAR_MAX_P.  n: elements per rank (0 is allowed: every call is a no-op).
- * steps: S in [ceil(log2 P), 2 ceil(log2 P)], or GAR_STEPS_BO / GAR_STEPS_LO.
+ * steps: S in [ceil(log2 P), 2 ceil(log2 P)], or GAR_STEPS_BO / GAR_STEPS_LO /
+ * GAR_STEPS_RING.
  * The block partition is the paper's V_j = (u_{0,j}, ..., u_{P-1,j}) (eq.
  * initial_data) with the first n mod P blocks one element longer.  Host-only: needs
  * no GPU.  *out is set only on success. */

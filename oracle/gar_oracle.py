@@ -75,7 +75,7 @@ __all__ = [
     "OPS", "DTYPES", "ceil_log2", "vector_counts", "block_bounds", "schedule_shape",
     "ExprTable", "Run", "simulate", "allreduce", "round_to_bf16", "is_bf16_exact",
     "column_reduce_exact", "kahan_sum_f64", "tree_string", "parse_tree",
-    "eval_tree", "cost_model_time", "optimal_steps", "group_ops",
+    "eval_tree", "cost_model_time", "optimal_steps", "group_ops", "simulate_ring",
 ]
 
 OPS = ("sum", "max", "min")
@@ -515,6 +515,98 @@ def simulate(P: int, n: int, steps: int, inputs=None, op: str = "sum",
     return run
 
 
+def simulate_ring(P: int, n: int, inputs=None, op: str = "sum", dtype: str = "f32",
+                  elements=None) -> Run:
+    """The Ring algorithm: the straightforward Allreduce of Sec. "Allreduce as
+    permutation composition" with the cyclic group, whose operator t_{i->0} reduces to the
+    generator t (x -> x + 1).  Reduction step i (i = 0..P-2): the partial vector at
+    placement i moves by t to placement i + 1 and is combined with the initial vector
+    t^{i+1} q_{i+1} there (eq. ring_reduce: own t^{i+1} q_{i+1} (+) received).  After P-1
+    steps placement P-1 holds q_Sigma; the distribution phase moves copies by t again,
+    P-1 more steps (2(P-1) in total, eq. naive_cost)."""
+    if op not in OPS:
+        raise ValueError(op)
+    if dtype not in DTYPES:
+        raise ValueError(dtype)
+    bounds = block_bounds(n, P)
+    block_len = [hi - lo for (lo, hi) in bounds]
+    ex = ExprTable()
+    itemsize, acc_itemsize = _ITEMSIZE[dtype], _ACC_ITEMSIZE[dtype]
+    if elements is None:
+        sel = [np.arange(lo, hi, dtype=np.int64) for (lo, hi) in bounds]
+    else:
+        elements = np.asarray(elements, dtype=np.int64)
+        sel = [elements[(elements >= lo) & (elements < hi)] for (lo, hi) in bounds]
+    have_values = inputs is not None
+    if have_values:
+        want = np.int32 if dtype == "i32" else np.float32
+        inputs = [np.asarray(v) for v in inputs]
+        for v in inputs:
+            if v.shape != (n,) or v.dtype != want:
+                raise ValueError(f"input must be shape ({n},) {want}")
+            if dtype == "bf16" and not is_bf16_exact(v):
+                raise ValueError("bf16 inputs must be exactly representable in bf16")
+    L = ceil_log2(P)
+    run = Run(P=P, n=n, steps=2 * (P - 1), L=L, r=0, K=1, op=op, dtype=dtype, exprs=ex,
+              outputs=None)
+    store = [dict() for _ in range(P)]
+    for x in range(P):
+        for k in range(P):
+            b = (x - k) % P
+            store[x][(k, ex.leaf(k))] = inputs[x][sel[b]].copy() if have_values else None
+    cur = (0, ex.leaf(0)) if P > 0 else None      # the partial q', at placement 0
+    for i in range(P - 1):
+        messages, inbox = [], [dict() for _ in range(P)]
+        for x in range(P):
+            dst = (x + 1) % P                      # operator t
+            b = (x - cur[0]) % P
+            sz = itemsize if ex.is_leaf(cur[1]) else acc_itemsize
+            messages.append((x, dst, [(cur, block_len[b], sz)]))
+            inbox[dst][((cur[0] + 1) % P, cur[1])] = store[x][cur]
+        run.log.append({"phase": "reduce", "i": i, "N": None, "d": -1, "tx": [cur],
+                        "messages": messages})
+        own = ((i + 1) % P, ex.leaf((i + 1) % P))
+        key = (own[0], ex.pair(own[1], cur[1]))
+        new_store = [dict() for _ in range(P)]
+        for x in range(P):
+            for k2, v in store[x].items():
+                if k2 != cur and k2 != own:
+                    new_store[x][k2] = v
+            recv = inbox[x][((cur[0] + 1) % P, cur[1])]
+            new_store[x][key] = _combine(op, store[x][own], recv) if have_values else None
+        store, cur = new_store, key
+        run.states.append([[cur]])
+        run.combines.append([key])
+    run.after_reduction = [cur] if P > 0 else []
+    at_place = {cur[0]: cur} if P > 0 else {}
+    if have_values and dtype == "bf16" and P > 0:
+        for x in range(P):
+            store[x][cur] = round_to_bf16(store[x][cur])
+    last = cur
+    for j in range(P - 1):
+        messages, inbox = [], [dict() for _ in range(P)]
+        for x in range(P):
+            dst = (x + 1) % P
+            b = (x - last[0]) % P
+            messages.append((x, dst, [(last, block_len[b], itemsize)]))
+            inbox[dst][((last[0] + 1) % P, last[1])] = store[x][last]
+        run.log.append({"phase": "distribute", "i": j, "N": None, "d": -1, "tx": [last],
+                        "messages": messages})
+        newkey = ((last[0] + 1) % P, last[1])
+        assert newkey[0] not in at_place
+        at_place[newkey[0]] = newkey
+        for x in range(P):
+            store[x][newkey] = inbox[x][newkey]
+        last = newkey
+    if P > 0:
+        assert sorted(at_place) == list(range(P))
+    run.out_key = [[at_place[(x - b) % P] for b in range(P)] for x in range(P)]
+    if have_values:
+        run.outputs = [np.concatenate([store[x][run.out_key[x][b]] for b in range(P)])
+                       if P else np.zeros(0) for x in range(P)]
+    return run
+
+
 def allreduce(inputs, steps: int, op: str = "sum", dtype: str = "f32", elements=None,
               group: str = "cyclic"):
     """MPI_Allreduce semantics (Sec. "Introduction"): every process ends with the
@@ -522,6 +614,8 @@ def allreduce(inputs, steps: int, op: str = "sum", dtype: str = "f32", elements=
     selected elements when ``elements`` is given)."""
     P = len(inputs)
     n = len(inputs[0]) if P else 0
+    if steps == "ring":
+        return simulate_ring(P, n, inputs=inputs, op=op, dtype=dtype, elements=elements).outputs
     return simulate(P, n, steps, inputs=inputs, op=op, dtype=dtype,
                     elements=elements, group=group).outputs
 

@@ -332,9 +332,15 @@ int gar_plan_create_group(gar_plan **out, int P, uint64_t n, int dtype, int op, 
   }
   const int L = ceil_log2(P);
   int S = steps;
+  const bool ring = steps == GAR_STEPS_RING;
+  if (ring && group != GAR_GROUP_CYCLIC) {
+    set_error("the Ring schedule uses the cyclic group");
+    return GAR_EINVAL;
+  }
   if (steps == GAR_STEPS_BO) S = 2 * L;
   if (steps == GAR_STEPS_LO) S = L;
-  if (S < L || S > 2 * L) {
+  if (ring) S = 2 * (P - 1);
+  if (!ring && (S < L || S > 2 * L)) {
     set_error("steps must be in [" + std::to_string(L) + ", " + std::to_string(2 * L) + "] for P=" +
               std::to_string(P));
     return GAR_EINVAL;
@@ -347,6 +353,7 @@ int gar_plan_create_group(gar_plan **out, int P, uint64_t n, int dtype, int op, 
   pl->op = op;
   pl->S = S;
   pl->group = group;
+  pl->ring = ring;
   int rc = build_plan(pl);
   if (rc) {
     delete pl;
@@ -389,6 +396,7 @@ int gar_plan_get_info(const gar_plan *pl, gar_plan_info *info) {
   info->n = pl->n;
   info->fused_combines = (int)pl->prog.a.size();
   info->group = pl->group;
+  info->ring = pl->ring ? 1 : 0;
   info->fused_width = pl->fused_width;
   if (pl->fused != nullptr && pl->fused->loaded) {
     info->fused_regs = pl->fused->regs;

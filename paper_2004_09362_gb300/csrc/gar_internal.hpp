@@ -75,6 +75,7 @@ constexpr int GAR_HOST_CHUNKS_MAX = 16;  // element chunks of the pipelined host
 struct gar_plan {
   int P = 0, L = 0, S = 0, r = 0, K = 0;
   int group = 0;                  // GAR_GROUP_CYCLIC or GAR_GROUP_XOR
+  bool ring = false;              // the Ring schedule (S = 2(P-1)) instead of S in [L, 2L]
   uint64_t n = 0;
   int dtype = 0, op = 0;
   uint64_t q = 0, rem = 0;        // block i has q + (i < rem) elements

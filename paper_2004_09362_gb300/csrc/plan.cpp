@@ -314,6 +314,78 @@ void build_fused(gar_plan *pl) {
     if (fp.origin[p] < 0) throw std::logic_error("placement without a result");
 }
 
+// The Ring (Sec. "Allreduce as permutation composition", cyclic group: the operator of
+// every step is the generator t, x -> x + 1).  Reduction step i moves the partial at
+// placement i to placement i + 1 and combines it there with the rank's own initial block
+// (eq. ring_reduce); distribution step j moves the copy at placement P-1+j on by one.
+// In place: step i writes placement i + 1 while the partner reads placement i.
+void build_ring(gar_plan *pl) {
+  const int P = pl->P;
+  const bool acc_is_elem = pl->dtype != GAR_BF16;
+  const Buf partial = acc_is_elem ? BUF_RANK : BUF_QP0;
+  for (int i = 0; i + 1 < P; ++i) {
+    const bool last = (i + 2 == P);
+    const Buf src = (i == 0) ? BUF_RANK : partial;
+    CommStep cs;
+    cs.phase = 0;
+    cs.i = i;
+    cs.N = 0;
+    cs.d = 1;
+    cs.partner = -1;
+    cs.tx = {i};
+    Launch ln;
+    ln.phase = 0;
+    ln.comm_step = (int)pl->comm.size();
+    ln.partner = -1;
+    ln.first_op = (int)pl->ops.size();
+    StepOp op = make_op(i, i + 1, src);
+    add_out(op, last ? BUF_RANK : partial, BUF_RANK);   // own initial block (+) received partial
+    pl->ops.push_back(op);
+    ln.nops = 1;
+    cs.msg_bytes = pl->n * (uint64_t)(src == BUF_RANK ? elem_size(pl->dtype) : acc_size(pl->dtype));
+    pl->comm.push_back(cs);
+    pl->launches.push_back(ln);
+  }
+  for (int j = 0; j + 1 < P; ++j) {
+    const int from = (P - 1 + j) % P, to = j;
+    CommStep cs;
+    cs.phase = 1;
+    cs.i = j;
+    cs.N = 0;
+    cs.d = 1;
+    cs.partner = -1;
+    cs.tx = {from};
+    Launch ln;
+    ln.phase = 1;
+    ln.comm_step = (int)pl->comm.size();
+    ln.partner = -1;
+    ln.first_op = (int)pl->ops.size();
+    StepOp op = make_op(from, to, BUF_RANK);
+    add_out(op, BUF_RANK, BUF_NONE);
+    pl->ops.push_back(op);
+    ln.nops = 1;
+    cs.msg_bytes = pl->n * (uint64_t)elem_size(pl->dtype);
+    pl->comm.push_back(cs);
+    pl->launches.push_back(ln);
+  }
+  for (const StepOp &op : pl->ops)
+    for (uint8_t b : {op.recv_buf, op.out0_buf, op.out0_own, op.out1_buf, op.out1_own})
+      if (b >= BUF_QP0) pl->ws_used[b - BUF_QP0] = true;
+  // fused program: the chain q_{P-1} (+) (... (+) (q_1 (+) q_0)), written to every rank
+  FusedProgram &fp = pl->prog;
+  fp = FusedProgram{};
+  fp.P = P;
+  fp.K = 1;
+  int v = 0;
+  for (int k = 1; k < P; ++k) {
+    fp.a.push_back(k);
+    fp.b.push_back(v);
+    v = P + (int)fp.a.size() - 1;
+  }
+  fp.out.push_back(v);
+  fp.origin.assign(P, 0);
+}
+
 }  // namespace
 
 int build_plan(gar_plan *pl) {
@@ -323,17 +395,26 @@ int build_plan(gar_plan *pl) {
   pl->N.push_back(P);
   while (pl->N.back() > 1) pl->N.push_back((pl->N.back() + 1) / 2);
   if ((int)pl->N.size() != pl->L + 1) return GAR_EINVAL;
-  pl->r = 2 * pl->L - pl->S;
-  if (pl->r < 0 || pl->r > pl->L) return GAR_EINVAL;
-  pl->K = pl->N[pl->L - pl->r];
+  if (pl->ring) {
+    pl->r = 0;
+    pl->K = 1;
+  } else {
+    pl->r = 2 * pl->L - pl->S;
+    if (pl->r < 0 || pl->r > pl->L) return GAR_EINVAL;
+    pl->K = pl->N[pl->L - pl->r];
+  }
   pl->q = pl->n / (uint64_t)P;
   pl->rem = pl->n % (uint64_t)P;
   pl->comm.clear();
   pl->ops.clear();
   pl->launches.clear();
   try {
-    build_step_faithful(pl);
-    build_fused(pl);
+    if (pl->ring) {
+      build_ring(pl);
+    } else {
+      build_step_faithful(pl);
+      build_fused(pl);
+    }
   } catch (const std::exception &e) {
     set_error(std::string("schedule builder: ") + e.what());
     return GAR_EINVAL;

@@ -396,6 +396,20 @@ def test_batched_mixed_groups():
                                           want[x].view(np.uint32))
 
 
+@pytest.mark.parametrize("P", [2, 3, 5, 8, 24])
+@pytest.mark.parametrize("mode", ["fused", "step", "persistent"])
+def test_ring_matches_oracle(P, mode):
+    """The Ring schedule (2(P-1) steps) bit for bit against the oracle's Ring."""
+    for (n, dtype) in [(2 * P + 3, "f32"), (2 * P + 3, "bf16"), (2 * P + 3, "i32"), (P * 4001 + 3, "f32")]:
+        t = _np_inputs(P, n, dtype, seed=29 * P + n)
+        host = _to_host_list(t, dtype)
+        plan = gar.gar_plan_create(P, n, dtype, "sum", gar.GAR_STEPS_RING)
+        got = _run(plan, t, mode)
+        _assert_same(got, G.allreduce(host, "ring", "sum", dtype), dtype, f"ring P={P} n={n} {dtype} {mode}")
+        if mode != "fused":
+            assert gar.gar_last_step_bytes(plan) == gar.gar_plan_bytes(plan)[1]
+
+
 # ---------------------------------------------------------------------------
 # Persistent step-faithful mode: one cooperative launch, bounded grid barriers
 # ---------------------------------------------------------------------------

@@ -584,3 +584,68 @@ def test_xor_group_coverage_bruteforce_and_traffic(P):
 def test_xor_group_needs_power_of_two():
     with pytest.raises(ValueError):
         G.simulate(6, 0, 4, group="xor")
+
+
+# ---------------------------------------------------------------------------
+# The Ring algorithm (Sec. "Allreduce as permutation composition", cyclic case)
+# ---------------------------------------------------------------------------
+
+def _textbook_ring(xs):
+    """Ring Allreduce as usually described: P-1 reduce-scatter steps in which rank x
+    passes its running partial of chunk (x - i) mod P to rank x + 1, which adds its own
+    chunk to it, then P-1 allgather steps passing the finished chunks on.  Written
+    independently of the oracle's schedule simulation."""
+    P, n = len(xs), len(xs[0])
+    bounds = G.block_bounds(n, P)
+    buf = [x.copy() for x in xs]
+    for i in range(P - 1):
+        new = [b.copy() for b in buf]
+        for x in range(P):
+            c = (x - i) % P
+            y = (x + 1) % P
+            lo, hi = bounds[c]
+            new[y][lo:hi] = buf[y][lo:hi] + buf[x][lo:hi]
+        buf = new
+    for i in range(P - 1):
+        new = [b.copy() for b in buf]
+        for x in range(P):
+            c = (x + 1 - i) % P
+            y = (x + 1) % P
+            lo, hi = bounds[c]
+            new[y][lo:hi] = buf[x][lo:hi]
+        buf = new
+    return buf
+
+
+@pytest.mark.parametrize("P", [2, 3, 5, 7, 8, 13, 24])
+def test_ring_equals_textbook_ring(P):
+    rng = np.random.default_rng(200 + P)
+    n = 3 * P + 2
+    xs = [(rng.standard_normal(n) * np.exp2(rng.integers(-20, 21, n))).astype(np.float32)
+          for _ in range(P)]
+    got = G.allreduce(xs, "ring", "sum", "f32")
+    want = _textbook_ring(xs)
+    for x in range(P):
+        np.testing.assert_array_equal(got[x].view(np.uint32), want[x].view(np.uint32))
+
+
+@pytest.mark.parametrize("P", [1, 2, 3, 4, 5, 9, 16, 31])
+def test_ring_steps_traffic_and_tree(P):
+    """2(P-1) steps, 2(P-1) blocks and P-1 combines per rank (eq. naive_cost); the
+    result is the chain of eq. ring_reduce: q_{P-1} (+) (... (+) (q_1 (+) q_0))."""
+    rng = np.random.default_rng(P)
+    n = 2 * P + 1
+    xs = [rng.integers(-1000, 1001, n).astype(np.int32) for _ in range(P)]
+    run = G.simulate_ring(P, n, inputs=xs, dtype="i32")
+    assert len(run.log) == 2 * (P - 1)
+    ref = G.column_reduce_exact(xs, "sum", "i32")
+    for o in run.outputs:
+        np.testing.assert_array_equal(o, ref)
+    for x in range(P):
+        assert run.message_blocks_per_rank(x) == 2 * (P - 1)
+    assert sum(len(c) for c in run.combines) == P - 1
+    if P >= 2:
+        chain = 0
+        for k in range(1, P):
+            chain = (k, chain)
+        assert run.exprs.tree(run.after_reduction[0][1]) == chain

@@ -298,3 +298,40 @@ def test_cost_model_matches_oracle():
                 assert gar.gar_optimal_steps(P, m, a, b, c) == G.optimal_steps(P, m, a, b, c)
     with pytest.raises(gar.GarError):
         gar.gar_cost_model(8, 2, 1.0, 1.0, 1.0, 1.0)
+
+
+@pytest.mark.parametrize("P", [1, 2, 3, 4, 5, 7, 8, 13, 24, 33])
+def test_ring_plan_matches_oracle(P):
+    """GAR_STEPS_RING: steps, partners, transmitted placements and bytes against the
+    oracle's Ring simulation; the op tables and the fused program reproduce its results
+    bit for bit on the CPU."""
+    rng = np.random.default_rng(500 + P)
+    n = 2 * P + 3
+    for dtype in ("f32", "bf16", "i32"):
+        plan = gar.gar_plan_create(P, n, dtype, "sum", gar.GAR_STEPS_RING)
+        run = G.simulate_ring(P, n, dtype=dtype)
+        info = plan.info()
+        assert info["ring"] == 1 and info["S"] == 2 * (P - 1) == len(run.log)
+        _ws, per_step, _S = gar.gar_plan_bytes(plan)
+        assert per_step == run.step_bytes()
+        for t, st in enumerate(run.log):
+            phase, partner, tx = gar.gar_plan_step(plan, t)
+            assert phase == (0 if st["phase"] == "reduce" else 1) and partner == -1
+            assert tx == [k[0] for k in st["tx"]]
+        if dtype == "i32":
+            xs = [rng.integers(-1000, 1001, n).astype(np.int32) for _ in range(P)]
+        else:
+            xs = [(rng.standard_normal(n) * np.exp2(rng.integers(-10, 11, n))).astype(np.float32)
+                  for _ in range(P)]
+            if dtype == "bf16":
+                xs = [G.round_to_bf16(v) for v in xs]
+        want = G.simulate_ring(P, n, inputs=xs, dtype=dtype).outputs
+        got = emulate_step_faithful(plan, xs, dtype, "sum")
+        for x in range(P):
+            np.testing.assert_array_equal(got[x].view(np.uint32), want[x].view(np.uint32))
+        if dtype == "f32":
+            got = emulate_fused(plan, xs, "sum")
+            for x in range(P):
+                np.testing.assert_array_equal(got[x].view(np.uint32), want[x].view(np.uint32))
+    with pytest.raises(gar.GarError):
+        gar.gar_plan_create_group(8, 10, "f32", "sum", gar.GAR_STEPS_RING, "xor")
