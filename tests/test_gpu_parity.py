@@ -168,6 +168,27 @@ def test_p127_bf16_reduced_n(mode):
         _assert_same(_run(plan, t, mode), G.allreduce(host, S, "sum", "bf16"), "bf16", f"S={S}")
 
 
+@pytest.mark.parametrize("P,n,dtype", [(32, 32 * 40000 + 13, "bf16"), (64, 1 << 20, "f32"),
+                                       (48, 48 * 2048 * 3 + 100, "i32")])
+def test_latency_optimal_mid_size_fused(P, n, dtype):
+    """Latency-optimal programs with P = 32..64 (hundreds of combines per element
+    position, every rank its own tree rotation) at sizes with ragged tails, checked on
+    sampled positions."""
+    t = _np_inputs(P, n, dtype, seed=P)
+    plan = gar.gar_plan_create(P, n, dtype, "sum", gar.GAR_STEPS_LO)
+    got = _run(plan, t, "fused")
+    idx = _sample(n, P, k=2048, seed=P)
+    full = [np.zeros(n, np.float32 if dtype != "i32" else np.int32) for _ in range(P)]
+    host = _to_host_list(t, dtype)
+    for x in range(P):
+        full[x][idx] = host[x][idx]
+    want = G.allreduce(full, G.ceil_log2(P), "sum", dtype, elements=idx)
+    gotl = _to_host_list(got, dtype)
+    for x in range(P):
+        g = gotl[x][idx].astype(want[x].dtype)
+        assert np.array_equal(_bits(g), _bits(want[x])), f"rank {x}"
+
+
 # ---------------------------------------------------------------------------
 # Recorded step bytes equal the schedule's predicted volume
 # ---------------------------------------------------------------------------
