@@ -110,6 +110,45 @@ def test_mid_size_chunked_step_kernel(P):
             assert rec == gar.gar_plan_bytes(plan)[1]
 
 
+@pytest.mark.parametrize("P", range(18, 41))
+@pytest.mark.parametrize("mode", ["fused", "step"])
+def test_every_p_to_40(P, mode):
+    """Every P up to 40 and every step count, fp32, ragged blocks."""
+    n = 4 * P + 3
+    t = _np_inputs(P, n, "f32", seed=P)
+    host = _to_host_list(t, "f32")
+    for S in _Ss(P):
+        plan = gar.gar_plan_create(P, n, "f32", "sum", S)
+        _assert_same(_run(plan, t, mode), G.allreduce(host, S, "sum", "f32"), "f32", f"P={P} S={S} {mode}")
+
+
+@pytest.mark.parametrize("mode", ["fused", "step", "persistent"])
+def test_cuda_graph_capture_and_replay(mode):
+    """After gar_plan_prepare, Allreduce calls can be captured into a CUDA graph; each
+    replay reduces the buffers' current contents."""
+    P, n, S = 7, 7 * 3000 + 5, 4
+    t = _np_inputs(P, n, "f32", seed=3)
+    plan = gar.gar_plan_create(P, n, "f32", "sum", S)
+    if mode != "fused":
+        gar.ensure_workspace(plan)
+    gar.gar_plan_prepare(plan, "fused" if mode == "fused" else "step")
+    store, view = _padded_device(t)
+    side = torch.cuda.Stream()
+    side.wait_stream(torch.cuda.current_stream())
+    graph = torch.cuda.CUDAGraph()
+    with torch.cuda.stream(side):
+        with torch.cuda.graph(graph, stream=side):
+            gar.gar_allreduce(plan, store, mode, side)
+    torch.cuda.current_stream().wait_stream(side)
+    host = _to_host_list(t, "f32")
+    for rep in range(2):
+        store[:, :n] = torch.from_numpy(np.stack(host)).to(DEV)
+        graph.replay()
+        torch.cuda.synchronize()
+        _assert_same(view.cpu(), G.allreduce(host, S, "sum", "f32"), "f32", f"graph replay {rep} {mode}")
+        host = [h * np.float32(0.5) for h in host]
+
+
 @pytest.mark.parametrize("op", ["max", "min"])
 @pytest.mark.parametrize("mode", ["fused", "step"])
 def test_small_max_min(op, mode):
