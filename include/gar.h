@@ -141,6 +141,7 @@ GAR_API int gar_plan_create_group(gar_plan **out, int P, uint64_t n, int dtype, 
  * no work using the plan is still running. */
 GAR_API void gar_plan_destroy(gar_plan *plan);
 
+/* Fills *info (see gar_plan_info).  Host-only. */
 GAR_API int gar_plan_get_info(const gar_plan *plan, gar_plan_info *info);
 
 /* Sizes.  workspace_bytes: device workspace step-faithful mode needs (0 when the
@@ -153,23 +154,26 @@ GAR_API int gar_plan_bytes(const gar_plan *plan, size_t *workspace_bytes,
                    uint64_t *msg_bytes_per_step, int *S);
 
 /* Schedule introspection (host-only).  For communication step t in [0, S):
- * phase = 0 (reduction) or 1 (distribution); partner = offset so that rank x
- * receives from rank (x + partner) mod P (reduction: +floor(N_i/2), eq. bo_dir_perms;
- * distribution: -floor(N_i/2)); placements[0..*count) = placements of the vectors
- * each rank transmits (eq. bo_tx_dist and its shifted forms).  placements may be
- * NULL to query the count; otherwise it must hold P entries. */
+ * phase = 0 (reduction) or 1 (distribution); partner: rank x receives from rank
+ * (x + partner) mod P in the cyclic group (reduction: +floor(N_i/2), eq. bo_dir_perms;
+ * distribution: -floor(N_i/2); the Ring: -1 in both phases) and from rank x XOR
+ * partner in the XOR group; placements[0..*count) = placements of the vectors each rank
+ * transmits (eq. bo_tx_dist and its shifted forms).  placements may be NULL to query
+ * the count; otherwise it must hold P entries. */
 GAR_API int gar_plan_step(const gar_plan *plan, int t, int *phase, int *partner,
                   int32_t *placements, int *count);
 
 /* origin[p] for p in [0, P): the result copy (0..K-1) that placement p receives in the
- * distribution phase.  Rank x's result for block b is placement (x - b) mod P. */
+ * distribution phase (end of Sec. "Bandwidth-optimal algorithm").  Rank x's result for
+ * block b is at placement (x - b) mod P (cyclic group) or x XOR b (XOR group). */
 GAR_API int gar_plan_origin(const gar_plan *plan, int32_t *origin);
 
 /* The fused-mode program: value ids 0..P-1 are the P contributions of an element
- * position rotated by its block b (id j = rank (b + j) mod P); combine k makes value
- * P + k = ops[2k] (+) ops[2k+1] (own, received).  outputs[s] (s < K) = value id of
- * result copy s.  Pass NULL arrays to query *nops; ops must hold 2 * *nops entries and
- * outputs K entries. */
+ * position in block b, contribution j coming from rank t_j(b) ((b + j) mod P, or b XOR j
+ * in the XOR group); combine k makes value P + k = ops[2k] (+) ops[2k+1] (own,
+ * received; eq. distr_vectors_combination).  outputs[s] (s < K) = value id of result
+ * copy s.  Pass NULL arrays to query *nops; ops must hold 2 * *nops entries and outputs
+ * K entries. */
 GAR_API int gar_plan_fused_program(const gar_plan *plan, int32_t *ops, int *nops, int32_t *outputs);
 
 /* The step-faithful op table (host-only, for inspection and tests).  Each op is 8
@@ -236,12 +240,13 @@ typedef struct {
 GAR_API int gar_allreduce_batched(gar_plan *const *plans, int nplans, const gar_batch_desc *desc,
                           int count, gar_stream_t stream);
 
-/* Outcome of the plan's most recent GAR_STEP_PERSISTENT Allreduce: waits for the stream
- * it ran on, then returns GAR_OK, GAR_ETIMEOUT if a grid-barrier wait gave up (the
- * results are then incomplete), or GAR_ECUDA.  GAR_OK if no persistent call ran. */
+/* Outcome of the plan's most recent GAR_STEP_PERSISTENT Allreduce (no counterpart in
+ * the paper: failure reporting of the bounded waits): waits for the stream it ran on,
+ * then returns GAR_OK, GAR_ETIMEOUT if a grid-barrier wait gave up (the results are then
+ * incomplete), or GAR_ECUDA.  GAR_OK if no persistent call ran. */
 GAR_API int gar_plan_status(gar_plan *plan);
 
-/* Barrier parameters of GAR_STEP_PERSISTENT.  spin_limit: polls (each an L2 round trip
+/* Barrier parameters of GAR_STEP_PERSISTENT (no counterpart in the paper).  spin_limit: polls (each an L2 round trip
  * plus a 64 ns sleep) a CTA makes at a grid barrier before it gives up (0 restores the
  * default, 2^20, roughly a second).
  * phantom: extra arrivals the barrier waits for beyond the launched CTAs -- nonzero
@@ -254,7 +259,9 @@ GAR_API int gar_plan_debug_barrier(gar_plan *plan, unsigned int phantom, unsigne
  * of that call. */
 GAR_API int gar_last_step_bytes(const gar_plan *plan, uint64_t *per_step);
 
+/* Name of a GAR_* status code (static string). */
 GAR_API const char *gar_strerror(int status);
+/* The calling thread's most recent error detail (valid until its next failing call). */
 GAR_API const char *gar_last_error(void);
 
 /* The paper's cost model (Sec. "Communication model": tau = alpha + beta m + gamma m per
