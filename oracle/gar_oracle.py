@@ -76,6 +76,7 @@ __all__ = [
     "ExprTable", "Run", "simulate", "allreduce", "round_to_bf16", "is_bf16_exact",
     "column_reduce_exact", "kahan_sum_f64", "tree_string", "parse_tree",
     "eval_tree", "cost_model_time", "optimal_steps", "group_ops", "simulate_ring",
+    "fold_sequence",
 ]
 
 OPS = ("sum", "max", "min")
@@ -126,13 +127,44 @@ def schedule_shape(P: int, steps: int) -> dict:
     """Step count S in [L, 2L] (abstract; Sec. "Moving towards latency-optimal
     version": S = 2 ceil(log P) - r, 0 <= r <= ceil(log P)).  Returns L, S, r and the
     number K of q_Sigma copies the reduction phase must end with (reading C7:
-    K = N_{L-r})."""
+    K = N_{L-r}).  Even S in (2L, 2(P-1)] selects the fold schedule (fold_sequence;
+    K = 1), the step counts toward the Ring that Sec. "Conclusion" leaves to future work
+    (reading C19)."""
     L = ceil_log2(P)
-    if not (L <= steps <= 2 * L):
-        raise ValueError(f"steps={steps} outside [{L}, {2 * L}] for P={P}")
-    r = 2 * L - steps
-    K = vector_counts(P)[L - r]
-    return {"P": P, "L": L, "S": steps, "r": r, "K": K}
+    if L <= steps <= 2 * L:
+        r = 2 * L - steps
+        K = vector_counts(P)[L - r]
+        return {"P": P, "L": L, "S": steps, "r": r, "K": K}
+    if steps > 2 * L and steps <= 2 * (P - 1) and steps % 2 == 0:
+        return {"P": P, "L": L, "S": steps, "r": 0, "K": 1}
+    raise ValueError(f"steps={steps} outside [{L}, {2 * L}] and not an even count up to "
+                     f"{2 * (P - 1)} for P={P}")
+
+
+def fold_sequence(P: int, F: int) -> list[int]:
+    """Vectors folded per reduction step for F steps (reading C19).  A step with N
+    vectors and fold f moves the vectors with index [N-f, N) by t^{-f} onto [N-2f, N-f)
+    and combines them there; f = floor(N/2) is the bandwidth-optimal step (eqs.
+    bo_tx_dist, bo_dir_perms), f = 1 moves one vector by the generator.  F = L gives the
+    bandwidth-optimal halving; F > L spreads the P-1 folds as evenly as the constraints
+    allow (1 <= f <= floor(N/2), and the remaining steps must still reach N = 1)."""
+    L = ceil_log2(P)
+    if not (L <= F <= max(P - 1, L)):
+        raise ValueError("F out of range")
+    if F == L:
+        Ns = vector_counts(P)
+        return [N // 2 for N in Ns[:-1]]
+    folds, N = [], P
+    for i in range(F):
+        r = F - i
+        lo = max(1, N - 2 ** (r - 1))
+        hi = min(N // 2, N - r)
+        want = -(-(N - 1) // r)          # ceil((N-1)/r): an even share of what is left
+        f = min(max(want, lo), hi)
+        folds.append(f)
+        N -= f
+    assert N == 1
+    return folds
 
 
 # ---------------------------------------------------------------------------
@@ -356,8 +388,17 @@ def simulate(P: int, n: int, steps: int, inputs=None, op: str = "sum",
         raise ValueError(dtype)
     gop, ginv = group_ops(P, group)
     shape = schedule_shape(P, steps)
+    if group == "xor" and steps > 2 * ceil_log2(P):
+        raise ValueError("fold schedules beyond 2L use the cyclic group")
     L, r, K = shape["L"], shape["r"], shape["K"]
-    Ns = vector_counts(P)
+    if steps > 2 * L:                       # fold schedule (reading C19)
+        folds = fold_sequence(P, steps // 2)
+    else:
+        folds = [N // 2 for N in vector_counts(P)[:-1]]
+    Ns = [P]
+    for f in folds:
+        Ns.append(Ns[-1] - f)
+    R = len(folds)                          # reduction steps
     bounds = block_bounds(n, P)
     block_len = [hi - lo for (lo, hi) in bounds]
     ex = ExprTable()
@@ -400,11 +441,11 @@ def simulate(P: int, n: int, steps: int, inputs=None, op: str = "sum",
     run = Run(P=P, n=n, steps=steps, L=L, r=r, K=K, op=op, dtype=dtype, exprs=ex,
               outputs=None)
 
-    # --- reduction phase: L steps
-    for i in range(L):
+    # --- reduction phase: R steps (L for S in [L, 2L])
+    for i in range(R):
         N = Ns[i]
-        d = N // 2            # operator t^{-floor(N_i/2)} (eq. bo_dir_perms)
-        c = N - d             # ceil(N_i/2)
+        d = folds[i]          # operator t^{-floor(N_i/2)} (eq. bo_dir_perms); t^{-f} for folds
+        c = N - d             # first transmitted index: ceil(N_i/2) when d = floor(N_i/2)
         # Q_TX,i of every shifted copy (eq. bo_tx_dist and its shifted form), each
         # distinct (placement, content) vector once.
         tx = []
@@ -440,8 +481,8 @@ def simulate(P: int, n: int, steps: int, inputs=None, op: str = "sum",
             q = sched[s]
             nq = []
             for k in range(c):
-                if k == 0 and N % 2 == 1:
-                    key = q[0]                 # q*: sits this step out
+                if k < N - 2 * d:
+                    key = q[k]                 # sits this step out (q* when N is odd)
                     for x in range(P):
                         new_store[x][key] = store[x][key]
                 else:
@@ -476,12 +517,12 @@ def simulate(P: int, n: int, steps: int, inputs=None, op: str = "sum",
                 key = at_place[s]
                 store[x][key] = round_to_bf16(store[x][key])
 
-    # --- distribution phase: reduction steps L-r-1 .. 0 reversed, no combination
-    for i in range(L - r - 1, -1, -1):
+    # --- distribution phase: reduction steps R-r-1 .. 0 reversed, no combination
+    for i in range(R - r - 1, -1, -1):
         N = Ns[i]
-        d = N // 2
+        d = folds[i]
         c = N - d
-        senders = list(range(N % 2, c))
+        senders = list(range(N - 2 * d, c))
         messages = []
         inbox = [dict() for _ in range(P)]
         for x in range(P):

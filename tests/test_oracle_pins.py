@@ -649,3 +649,73 @@ def test_ring_steps_traffic_and_tree(P):
         for k in range(1, P):
             chain = (k, chain)
         assert run.exprs.tree(run.after_reduction[0][1]) == chain
+
+
+# ---------------------------------------------------------------------------
+# Step counts beyond 2L: fold schedules toward the Ring (reading C19)
+# ---------------------------------------------------------------------------
+
+def _fold_cases():
+    out = []
+    for P in list(range(3, 41)) + [64, 127]:
+        L = G.ceil_log2(P)
+        Ss = list(range(2 * L + 2, 2 * (P - 1) + 1, 2))
+        if P > 40:
+            Ss = Ss[:3] + Ss[-2:]
+        out += [(P, S) for S in Ss]
+    return out
+
+
+@pytest.mark.parametrize("P,S", _fold_cases())
+def test_fold_schedule(P, S):
+    """Every even step count from 2L to 2(P-1): S steps; bandwidth-optimal traffic of
+    2(P-1) blocks per rank (eq. bo_cost's volume) whatever S; step i moves f_i <=
+    floor(N_i/2) blocks to rank x - f_i; every result covers every rank once; int32
+    results are the column sums; all ranks hold identical bits (one result copy)."""
+    L = G.ceil_log2(P)
+    F = S // 2
+    folds = G.fold_sequence(P, F)
+    assert len(folds) == F and sum(folds) == P - 1
+    N = P
+    for f in folds:
+        assert 1 <= f <= N // 2
+        N -= f
+    rng = np.random.default_rng(P * 100 + S)
+    n = 2 * P + 3
+    xs = [rng.integers(-1000, 1001, n).astype(np.int32) for _ in range(P)]
+    run = G.simulate(P, n, S, inputs=xs, dtype="i32")
+    assert len(run.log) == S and run.K == 1
+    ref = G.column_reduce_exact(xs, "sum", "i32")
+    for o in run.outputs:
+        np.testing.assert_array_equal(o, ref)
+    for x in range(P):
+        assert run.message_blocks_per_rank(x) == 2 * (P - 1)
+    red = [st for st in run.log if st["phase"] == "reduce"]
+    for st, f in zip(red, folds):
+        assert len(st["tx"]) == f
+        for (src, dst, _items) in st["messages"]:
+            assert dst == (src - f) % P
+    key = run.after_reduction[0]
+    assert sorted(run.exprs.leaves(key[1])) == list(range(P))
+    fx = [(rng.standard_normal(n) * np.exp2(rng.integers(-12, 13, n))).astype(np.float32)
+          for _ in range(P)]
+    outs = G.allreduce(fx, S, "sum", "f32")
+    for x in range(1, P):
+        np.testing.assert_array_equal(outs[x].view(np.uint32), outs[0].view(np.uint32))
+
+
+def test_fold_schedule_ends():
+    """F = L folds are the bandwidth-optimal halving; S = 2(P-1) folds one vector per step
+    and reduces to the chain q_0 (+) (q_1 (+) (... (+) (q_{P-2} (+) q_{P-1})))."""
+    for P in (5, 8, 13):
+        L = G.ceil_log2(P)
+        assert G.fold_sequence(P, L) == [N // 2 for N in G.vector_counts(P)[:-1]]
+        run = G.simulate(P, 0, 2 * (P - 1))
+        chain = P - 1
+        for k in range(P - 2, -1, -1):
+            chain = (k, chain)
+        assert run.exprs.tree(run.after_reduction[0][1]) == chain
+    with pytest.raises(ValueError):
+        G.simulate(8, 0, 9)                      # odd S beyond 2L
+    with pytest.raises(ValueError):
+        G.simulate(8, 0, 16)                     # beyond 2(P-1)
