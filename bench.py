@@ -284,7 +284,8 @@ def run_ours(args):
             bytes_step = _step_dram_bytes(gar, plan, P, n, wl.dtype)
         kernel_desc = (f"{args.mode} P{P} S{S} {wl.dtype} {args.op}"
                        + (f" W{info['fused_width']} regs{info['fused_regs']}" if args.mode == "fused" else ""))
-        sched = "bandwidth-optimal" if S == 2 * _l(P) else ("latency-optimal" if S == _l(P) else "intermediate")
+        sched = ("bandwidth-optimal" if S == 2 * _l(P) else "latency-optimal" if S == _l(P)
+                 else "fold" if S > 2 * _l(P) else "intermediate")
         config = {"workload": args.workload, "P": P, "n_per_rank": n,
                   "bytes_per_rank": n * (2 if wl.dtype == "bf16" else 4), "steps_S": S,
                   "schedule": sched, "mode": args.mode, "op": args.op,
@@ -510,20 +511,25 @@ def measure_rows(gar, gar_inputs, stream, hbm_peak):
     del flat, out
     torch.cuda.empty_cache()
     rows["groups_p64_4mib_f32"] = groups_row(gar, gar_inputs, stream, hbm_peak)
-    rows["ring_vs_bo_p24_64mib_f32"] = ring_row(gar, gar_inputs, stream, hbm_peak)
+    rows["step_range_p24_64mib_f32"] = step_range_row(gar, gar_inputs, stream, hbm_peak)
     rows["cost_model_p127_bf16_step"] = cost_model_row(gar, gar_inputs, stream)
     return rows
 
 
-def ring_row(gar, gar_inputs, stream, hbm_peak):
-    """The Ring (2(P-1) steps, the far end of the paper's step range) against the
-    bandwidth-optimal schedule (2L steps) on the headline workload, both modes."""
+def step_range_row(gar, gar_inputs, stream, hbm_peak):
+    """The whole step range on the headline workload, both modes: bandwidth-optimal
+    (2L steps), fold schedules from 2L + 2 to 2(P-1) steps (the fold of 2(P-1) steps
+    moves one vector per step), and the Ring (2(P-1) steps, every step by t)."""
     import torch
     wl = gar_inputs.WORKLOADS[HEADLINE]
     P, n = wl.P, wl.n
     inp = gar_inputs.rank_inputs(P, n, "f32", wl.dist, wl.seed, device="cuda")
+    L = _l(P)
+    scheds = [("bandwidth_optimal", gar.GAR_STEPS_BO)]
+    scheds += [(f"fold_S{S}", S) for S in (2 * L + 2, 16, 22, 30, 2 * (P - 1))]
+    scheds += [("ring", gar.GAR_STEPS_RING)]
     out = {}
-    for name, steps in (("ring", gar.GAR_STEPS_RING), ("bandwidth_optimal", gar.GAR_STEPS_BO)):
+    for name, steps in scheds:
         plan = gar.gar_plan_create(P, n, "f32", "sum", steps)
         gar.gar_plan_prepare(plan, "step")
         gar.gar_plan_prepare(plan, "fused")

@@ -124,7 +124,11 @@ typedef struct {
 /* Creates a schedule for P virtual ranks of n elements each.
  * P: 1..GAR_MAX_P.  n: elements per rank (0 is allowed: every call is a no-op).
  * steps: S in [ceil(log2 P), 2 ceil(log2 P)], or GAR_STEPS_BO / GAR_STEPS_LO /
- * GAR_STEPS_RING.
+ * GAR_STEPS_RING, or an even S in (2 ceil(log2 P), 2(P-1)] (cyclic group): a fold
+ * schedule, which generalizes the bandwidth-optimal step from folding floor(N_i/2)
+ * vectors to folding f_i <= floor(N_i/2) of them by t^{-f_i}, with the P-1 folds spread
+ * evenly over S/2 steps -- every such S moves the bandwidth-optimal 2(P-1) blocks per
+ * rank in smaller pieces (the step counts Sec. "Conclusion" leaves to future work).
  * The block partition is the paper's V_j = (u_{0,j}, ..., u_{P-1,j}) (eq.
  * initial_data) with the first n mod P blocks one element longer.  Host-only: needs
  * no GPU.  *out is set only on success. */

@@ -340,9 +340,14 @@ int gar_plan_create_group(gar_plan **out, int P, uint64_t n, int dtype, int op, 
   if (steps == GAR_STEPS_BO) S = 2 * L;
   if (steps == GAR_STEPS_LO) S = L;
   if (ring) S = 2 * (P - 1);
-  if (!ring && (S < L || S > 2 * L)) {
-    set_error("steps must be in [" + std::to_string(L) + ", " + std::to_string(2 * L) + "] for P=" +
-              std::to_string(P));
+  const bool folded = !ring && S > 2 * L && S <= 2 * (P - 1) && S % 2 == 0;
+  if (folded && group != GAR_GROUP_CYCLIC) {
+    set_error("step counts beyond 2L use the cyclic group");
+    return GAR_EINVAL;
+  }
+  if (!ring && !folded && (S < L || S > 2 * L)) {
+    set_error("steps must be in [" + std::to_string(L) + ", " + std::to_string(2 * L) +
+              "] or even up to " + std::to_string(2 * (P - 1)) + " for P=" + std::to_string(P));
     return GAR_EINVAL;
   }
   gar_plan *pl = new (std::nothrow) gar_plan();

@@ -76,6 +76,7 @@ struct gar_plan {
   int P = 0, L = 0, S = 0, r = 0, K = 0;
   int group = 0;                  // GAR_GROUP_CYCLIC or GAR_GROUP_XOR
   bool ring = false;              // the Ring schedule (S = 2(P-1)) instead of S in [L, 2L]
+  std::vector<int> folds;         // fold schedule (S > 2L): vectors folded per reduction step
   uint64_t n = 0;
   int dtype = 0, op = 0;
   uint64_t q = 0, rem = 0;        // block i has q + (i < rem) elements

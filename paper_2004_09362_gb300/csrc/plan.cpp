@@ -314,6 +314,112 @@ void build_fused(gar_plan *pl) {
     if (fp.origin[p] < 0) throw std::logic_error("placement without a result");
 }
 
+// Fold counts for F reduction steps (F > L): a step with N vectors folds f of them, the
+// ones with index [N-f, N), by t^{-f} onto [N-2f, N-f); f = floor(N/2) is the
+// bandwidth-optimal step.  The P-1 folds are spread as evenly as 1 <= f <= floor(N/2)
+// and reachability (the remaining steps, halving, must still get to N = 1) allow.
+std::vector<int> fold_counts(int P, int F) {
+  std::vector<int> folds;
+  int N = P;
+  for (int i = 0; i < F; ++i) {
+    const int r = F - i;
+    const long long pow2 = (r - 1 >= 31) ? (1LL << 31) : (1LL << (r - 1));
+    const int lo = (int)std::max<long long>(1, (long long)N - pow2);
+    const int hi = std::min(N / 2, N - r);
+    const int want = (N - 1 + r - 1) / r;  // ceil((N - 1) / r)
+    const int f = std::min(std::max(want, lo), hi);
+    folds.push_back(f);
+    N -= f;
+  }
+  if (N != 1) throw std::logic_error("fold schedule does not end with one vector");
+  return folds;
+}
+
+// Fold schedule (S = 2F > 2L, one result copy): step-faithful ops run in place like the
+// bandwidth-optimal schedule (transmitted [N-f, N) and combined [N-2f, N-f) placements
+// never overlap); placements [0, N-2f) sit the step out.  With a wider accumulation type
+// (bf16 -> fp32) a placement keeps its input in the rank buffer, and is sent in the
+// element type, until it is first combined; the combination lands in the fp32 slice.
+void build_folds(gar_plan *pl) {
+  const int P = pl->P;
+  const int F = (int)pl->folds.size();
+  const Buf inplace = pl->dtype != GAR_BF16 ? BUF_RANK : BUF_QP0;
+  std::vector<int> Ns{P};
+  for (int f : pl->folds) Ns.push_back(Ns.back() - f);
+  std::vector<Buf> loc(P, BUF_RANK);  // where each placement's vector lives now
+  for (int i = 0; i < F; ++i) {
+    const int N = Ns[i], f = pl->folds[i];
+    const bool last = (i == F - 1);
+    CommStep cs;
+    cs.phase = 0;
+    cs.i = i;
+    cs.N = N;
+    cs.d = f;
+    cs.partner = f;
+    cs.msg_bytes = 0;
+    Launch ln;
+    ln.phase = 0;
+    ln.comm_step = (int)pl->comm.size();
+    ln.partner = f;
+    ln.first_op = (int)pl->ops.size();
+    for (int p = N - f; p < N; ++p) {
+      cs.tx.push_back(p);
+      StepOp op = make_op(p, p - f, loc[p]);
+      add_out(op, last ? BUF_RANK : inplace, loc[p - f]);
+      pl->ops.push_back(op);
+      cs.msg_bytes += (uint64_t)pl->n *
+                      (uint64_t)(loc[p] == BUF_RANK ? elem_size(pl->dtype) : acc_size(pl->dtype));
+    }
+    for (int p = N - 2 * f; p < N - f; ++p) loc[p] = inplace;
+    ln.nops = (int)pl->ops.size() - ln.first_op;
+    pl->comm.push_back(cs);
+    pl->launches.push_back(ln);
+  }
+  for (int i = F - 1; i >= 0; --i) {
+    const int N = Ns[i], f = pl->folds[i];
+    CommStep cs;
+    cs.phase = 1;
+    cs.i = i;
+    cs.N = N;
+    cs.d = f;
+    cs.partner = -f;
+    Launch ln;
+    ln.phase = 1;
+    ln.comm_step = (int)pl->comm.size();
+    ln.partner = -f;
+    ln.first_op = (int)pl->ops.size();
+    for (int p = N - 2 * f; p < N - f; ++p) {
+      cs.tx.push_back(p);
+      StepOp op = make_op(p, p + f, BUF_RANK);
+      add_out(op, BUF_RANK, BUF_NONE);
+      pl->ops.push_back(op);
+    }
+    ln.nops = (int)pl->ops.size() - ln.first_op;
+    cs.msg_bytes = (uint64_t)f * pl->n * (uint64_t)elem_size(pl->dtype);
+    pl->comm.push_back(cs);
+    pl->launches.push_back(ln);
+  }
+  for (const StepOp &op : pl->ops)
+    for (uint8_t b : {op.recv_buf, op.out0_buf, op.out0_own, op.out1_buf, op.out1_own})
+      if (b >= BUF_QP0) pl->ws_used[b - BUF_QP0] = true;
+  FusedProgram &fp = pl->prog;
+  fp = FusedProgram{};
+  fp.P = P;
+  fp.K = 1;
+  std::vector<int> qp(P);
+  for (int p = 0; p < P; ++p) qp[p] = p;
+  for (int i = 0; i < F; ++i) {
+    const int N = Ns[i], f = pl->folds[i];
+    for (int k = N - 2 * f; k < N - f; ++k) {
+      fp.a.push_back(qp[k]);
+      fp.b.push_back(qp[k + f]);
+      qp[k] = P + (int)fp.a.size() - 1;
+    }
+  }
+  fp.out.push_back(qp[0]);
+  fp.origin.assign(P, 0);
+}
+
 // The Ring (Sec. "Allreduce as permutation composition", cyclic group: the operator of
 // every step is the generator t, x -> x + 1).  Reduction step i moves the partial at
 // placement i to placement i + 1 and combines it there with the rank's own initial block
@@ -398,6 +504,15 @@ int build_plan(gar_plan *pl) {
   if (pl->ring) {
     pl->r = 0;
     pl->K = 1;
+  } else if (pl->S > 2 * pl->L) {
+    pl->r = 0;
+    pl->K = 1;
+    try {
+      pl->folds = fold_counts(P, pl->S / 2);
+    } catch (const std::exception &e) {
+      set_error(std::string("schedule builder: ") + e.what());
+      return GAR_EINVAL;
+    }
   } else {
     pl->r = 2 * pl->L - pl->S;
     if (pl->r < 0 || pl->r > pl->L) return GAR_EINVAL;
@@ -411,6 +526,8 @@ int build_plan(gar_plan *pl) {
   try {
     if (pl->ring) {
       build_ring(pl);
+    } else if (!pl->folds.empty()) {
+      build_folds(pl);
     } else {
       build_step_faithful(pl);
       build_fused(pl);

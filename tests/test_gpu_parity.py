@@ -273,18 +273,22 @@ def _tree_bound_check(got_rows, inp, L, dtype):
         assert bool((err <= tol + 1e-30).all()), f"rank {r}: max excess {(err - tol).max().item()}"
 
 
+@pytest.mark.parametrize("S", [10, 22, 46])
 @pytest.mark.parametrize("mode", ["fused", "step"])
-def test_full_p24_64mib(mode):
+def test_full_p24_64mib(S, mode):
+    """The 24 x 64 MiB fp32 workload: bandwidth-optimal (S = 10) and two fold schedules
+    (S = 22, and S = 46 = 2(P-1), one vector folded per step)."""
     wl = gar_inputs.WORKLOADS["p24_64mib_f32"]
     P, n = wl.P, wl.n
     inp = gar_inputs.rank_inputs(P, n, wl.dtype, wl.dist, wl.seed, device=DEV)
     buf = inp.clone()
-    plan = gar.gar_plan_create(P, n, "f32", "sum", 10)
+    plan = gar.gar_plan_create(P, n, "f32", "sum", S)
     gar.gar_allreduce(plan, buf, mode)
     torch.cuda.synchronize()
-    # bandwidth-optimal: every rank holds identical bits
+    # one result copy: every rank holds identical bits
     assert bool((buf == buf[0:1]).all())
-    _tree_bound_check(buf, inp, 5, "f32")
+    # the result tree's depth is the number of reduction steps
+    _tree_bound_check(buf, inp, S // 2, "f32")
     idx = _sample(n, P)
     host_in = [inp[x, torch.from_numpy(idx).to(DEV)].cpu().numpy() for x in range(P)]
     # oracle on the sampled element positions: rebuild full-length vectors lazily by
@@ -292,7 +296,7 @@ def test_full_p24_64mib(mode):
     full = [np.zeros(n, np.float32) for _ in range(P)]
     for x in range(P):
         full[x][idx] = host_in[x]
-    want = G.allreduce(full, 10, "sum", "f32", elements=idx)
+    want = G.allreduce(full, S, "sum", "f32", elements=idx)
     got = buf[:, torch.from_numpy(idx).to(DEV)].cpu().numpy()
     for x in range(P):
         np.testing.assert_array_equal(got[x].view(np.uint32), want[x].view(np.uint32))
@@ -468,6 +472,33 @@ def test_ring_matches_oracle(P, mode):
         _assert_same(got, G.allreduce(host, "ring", "sum", dtype), dtype, f"ring P={P} n={n} {dtype} {mode}")
         if mode != "fused":
             assert gar.gar_last_step_bytes(plan) == gar.gar_plan_bytes(plan)[1]
+
+
+def _fold_Ss(P):
+    L = G.ceil_log2(P)
+    return list(range(2 * L + 2, 2 * (P - 1) + 1, 2))
+
+
+@pytest.mark.parametrize("P", [4, 5, 7, 8, 13, 24])
+@pytest.mark.parametrize("mode", ["fused", "step", "persistent"])
+def test_fold_schedules_match_oracle(P, mode):
+    """Fold schedules (every even S from 2L+2 to 2(P-1)) bit for bit against the oracle:
+    ragged small blocks in three types and with max, mid-size blocks (chunked step
+    launch) in fp32 and bf16; recorded step bytes equal the prediction."""
+    cases = [(2 * P + 3, "f32", "sum"), (2 * P + 3, "bf16", "sum"), (2 * P + 3, "i32", "sum"),
+             (2 * P + 3, "f32", "max"), (P * 4001 + 3, "f32", "sum"), (P * 2001 + 5, "bf16", "sum")]
+    for (n, dtype, op) in cases:
+        t = _np_inputs(P, n, dtype, seed=41 * P + n)
+        host = _to_host_list(t, dtype)
+        for S in _fold_Ss(P):
+            plan = gar.gar_plan_create(P, n, dtype, op, S)
+            got = _run(plan, t, mode)
+            _assert_same(got, G.allreduce(host, S, op, dtype), dtype,
+                         f"fold P={P} n={n} {dtype} {op} S={S} {mode}")
+            if mode != "fused":
+                assert gar.gar_last_step_bytes(plan) == gar.gar_plan_bytes(plan)[1]
+            if mode == "persistent":
+                assert gar.gar_plan_status(plan) == 0
 
 
 # ---------------------------------------------------------------------------

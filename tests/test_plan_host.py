@@ -50,6 +50,10 @@ def _cases():
         L = G.ceil_log2(P)
         for S in range(L, 2 * L + 1):
             out.append((P, S, "xor"))
+    for P in list(range(4, 34)) + [64, 127]:      # fold schedules: even S in (2L, 2(P-1)]
+        L = G.ceil_log2(P)
+        for S in range(2 * L + 2, 2 * (P - 1) + 1, 2):
+            out.append((P, S, "cyclic"))
     return out
 
 
@@ -221,6 +225,51 @@ def test_fused_program_reproduces_oracle(P, group):
             want = G.allreduce(xs, S, op, "f32", group=group)
             for x in range(P):
                 np.testing.assert_array_equal(got[x].view(np.uint32), want[x].view(np.uint32))
+
+
+@pytest.mark.parametrize("P", list(range(4, 18)) + [24, 33])
+def test_fold_tables_reproduce_oracle(P):
+    """Fold schedules (every even S from 2L+2 to 2(P-1)): the fold counts equal the
+    oracle's, and the step-faithful op tables and the fused program reproduce its
+    results bit for bit (bf16 sends a never-combined placement in bf16)."""
+    rng = np.random.default_rng(700 + P)
+    L = G.ceil_log2(P)
+    for n in sorted({P - 1, 2 * P + 3}):
+        for dtype in ("f32", "i32", "bf16"):
+            if dtype == "i32":
+                xs = [rng.integers(-1000, 1001, n).astype(np.int32) for _ in range(P)]
+            else:
+                xs = [(rng.standard_normal(n) * np.exp2(rng.integers(-10, 11, n))).astype(np.float32)
+                      for _ in range(P)]
+                if dtype == "bf16":
+                    xs = [G.round_to_bf16(v) for v in xs]
+            for S in range(2 * L + 2, 2 * (P - 1) + 1, 2):
+                plan = gar.gar_plan_create(P, n, dtype, "sum", S)
+                info = plan.info()
+                assert (info["S"], info["K"], info["r"], info["ring"]) == (S, 1, 0, 0)
+                assert [len(gar.gar_plan_step(plan, t)[2]) for t in range(S // 2)] == \
+                    G.fold_sequence(P, S // 2)
+                want = G.allreduce(xs, S, "sum", dtype)
+                got = emulate_step_faithful(plan, xs, dtype, "sum")
+                for x in range(P):
+                    np.testing.assert_array_equal(got[x].view(np.uint32), want[x].view(np.uint32))
+                if dtype == "f32":
+                    got = emulate_fused(plan, xs, "sum")
+                    for x in range(P):
+                        np.testing.assert_array_equal(got[x].view(np.uint32), want[x].view(np.uint32))
+                if dtype != "bf16":
+                    ws, _, _ = gar.gar_plan_bytes(plan)
+                    assert ws == 0                # in place, like bandwidth-optimal
+
+
+def test_fold_argument_errors():
+    with pytest.raises(gar.GarError):
+        gar.gar_plan_create(24, 10, steps=13)                  # odd S beyond 2L
+    with pytest.raises(gar.GarError):
+        gar.gar_plan_create(24, 10, steps=48)                  # beyond 2(P-1)
+    with pytest.raises(gar.GarError):
+        gar.gar_plan_create_group(16, 10, steps=10, group="xor")
+    assert gar.gar_plan_create(24, 10, steps=46).info()["S"] == 46
 
 
 def test_workspace_sizes():
