@@ -520,7 +520,7 @@ def measure_rows(gar, gar_inputs, stream, hbm_peak):
                                    [flat.data_ptr() + o * es for (_P, o) in layout],
                                    [out.data_ptr() + o * es for (_P, o) in layout])
         # 361 MB per call > 129 MB L2: back-to-back calls need no flush
-        ms = _time_loop(lambda: gar.gar_allreduce_batched(plans, desc, cfg["count"], stream), 20, 3,
+        ms = _time_loop(lambda: gar.gar_allreduce_batched(plans, desc, cfg["count"], stream), 50, 5,
                         stream)
         nbytes = 2 * flat.numel() * es
         rows[f"batched_65536x425B_{op}"] = {

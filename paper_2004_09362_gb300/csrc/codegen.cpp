@@ -414,9 +414,15 @@ CodegenResult generate_batched_source(const std::vector<const gar_plan *> &plans
   s += "  const gar_u64 per = nvec + (GAR_N - nvec * GAR_W);\n";
   s += "  const gar_u64 total = a.count * per;\n";
   s += "  const gar_u64 stride = (gar_u64)gridDim.x * blockDim.x;\n";
-  s += "  for (gar_u64 g = (gar_u64)blockIdx.x * blockDim.x + threadIdx.x; g < total; g += stride) {\n";
+  // A thread's next descriptor is loaded before its current item's contributions, so
+  // with fewer threads than items the descriptor latency overlaps the data loads.
+  s += "  gar_u64 g = (gar_u64)blockIdx.x * blockDim.x + threadIdx.x;\n";
+  s += "  if (g >= total) return;\n";
+  s += "  gar_desc dn = a.desc[g / per];\n";
+  s += "  for (; g < total; g += stride) {\n";
   s += "    const gar_u64 i = g / per, v = g - i * per;\n";
-  s += "    const gar_desc d = a.desc[i];\n";
+  s += "    const gar_desc d = dn;\n";
+  s += "    if (g + stride < total) dn = a.desc[(g + stride) / per];\n";
   s += "    const gar_io *in = (const gar_io *)d.in;\n";
   s += "    gar_io *out = (gar_io *)d.out;\n";
   s += "    const bool aligned = (((gar_u64)in | (gar_u64)out) & (GAR_W * sizeof(gar_io) - 1)) == 0;\n";
