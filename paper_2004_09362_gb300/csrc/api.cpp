@@ -80,9 +80,10 @@ int prepare_step_faithful(gar_plan *pl) {
     if (e != cudaSuccess) return cuda_fail(e, "cudaMemset(barrier state)");
   }
   if (pl->d_step_bytes == nullptr && pl->S > 0) {
-    cudaError_t e = cudaMalloc(&pl->d_step_bytes, pl->S * sizeof(unsigned long long));
+    const size_t cbytes = (size_t)pl->S * STEP_BYTE_SLOTS * sizeof(unsigned long long);
+    cudaError_t e = cudaMalloc(&pl->d_step_bytes, cbytes);
     if (e != cudaSuccess) return cuda_fail(e, "cudaMalloc(step counters)");
-    e = cudaMemset(pl->d_step_bytes, 0, pl->S * sizeof(unsigned long long));
+    e = cudaMemset(pl->d_step_bytes, 0, cbytes);
     if (e != cudaSuccess) return cuda_fail(e, "cudaMemset(step counters)");
   }
   return GAR_OK;
@@ -270,7 +271,8 @@ int run_step_faithful(gar_plan *pl, void *const *rank, gar_stream_t stream, bool
       return GAR_ENOWS;
     }
   }
-  cudaError_t e = cudaMemsetAsync(pl->d_step_bytes, 0, pl->S * sizeof(unsigned long long),
+  cudaError_t e = cudaMemsetAsync(pl->d_step_bytes, 0,
+                                  (size_t)pl->S * STEP_BYTE_SLOTS * sizeof(unsigned long long),
                                   (cudaStream_t)stream);
   if (e != cudaSuccess) return cuda_fail(e, "cudaMemsetAsync(step counters)");
   if (persistent) {
@@ -626,11 +628,15 @@ int gar_last_step_bytes(const gar_plan *pl, uint64_t *per_step) {
   }
   cudaError_t e = cudaStreamSynchronize((cudaStream_t)pl->last_stream);
   if (e != cudaSuccess) return cuda_fail(e, "cudaStreamSynchronize");
-  std::vector<unsigned long long> tmp(pl->S);
-  e = cudaMemcpy(tmp.data(), pl->d_step_bytes, pl->S * sizeof(unsigned long long),
+  std::vector<unsigned long long> tmp((size_t)pl->S * STEP_BYTE_SLOTS);
+  e = cudaMemcpy(tmp.data(), pl->d_step_bytes, tmp.size() * sizeof(unsigned long long),
                  cudaMemcpyDeviceToHost);
   if (e != cudaSuccess) return cuda_fail(e, "cudaMemcpy(step counters)");
-  for (int t = 0; t < pl->S; ++t) per_step[t] = tmp[t];
+  for (int t = 0; t < pl->S; ++t) {
+    uint64_t sum = 0;
+    for (int k = 0; k < STEP_BYTE_SLOTS; ++k) sum += tmp[(size_t)t * STEP_BYTE_SLOTS + k];
+    per_step[t] = sum;
+  }
   return GAR_OK;
 }
 

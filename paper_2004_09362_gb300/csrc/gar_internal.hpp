@@ -20,6 +20,10 @@ enum Buf : uint8_t {
   BUF_QS = 4     // q* slots (accumulation type)
 };
 constexpr int NUM_WS_BUFS = 3;  // QP0, QP1, QS
+// Each communication step's byte counter is spread over this many device slots (warps
+// add to slot (global warp index mod STEP_BYTE_SLOTS)); the reader sums them.  One
+// shared counter serialised ~10^5 same-address atomics per launch at L2.
+constexpr int STEP_BYTE_SLOTS = 32;
 
 // One block operation of a step-faithful launch, identical for every rank x.  With
 // b = (x - dst_place) mod P (the block index, which a move never changes):
