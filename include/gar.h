@@ -61,7 +61,12 @@ enum { GAR_SUM = 0, GAR_MAX = 1, GAR_MIN = 2 };
  *   gar_plan_bytes; records the bytes read from partners per step.
  * GAR_FUSED: one launch for the whole Allreduce; per element position the P
  *   contributions are loaded once, the reduction program that the schedule induces
- *   runs in registers, and every rank's result is written once.
+ *   runs in registers, and every rank's result is written once.  The program becomes
+ *   straight-line code compiled at run time, so fused mode takes programs of at most
+ *   GAR_FUSED_MAX_OPS operations (combines + P loads + P stores; the compile of the
+ *   largest takes about a minute on one core, and it grows faster than linearly).
+ *   Larger programs -- latency-optimal schedules at a few hundred ranks and up -- make
+ *   every fused call return GAR_EINVAL; GAR_STEP_FAITHFUL runs any plan.
  * GAR_STEP_PERSISTENT: the step-faithful schedule in one cooperative launch; a
  *   grid-wide barrier separates the steps instead of a kernel boundary.  Every barrier
  *   wait is bounded (gar_plan_debug_barrier): a CTA that waits too long records a
@@ -69,6 +74,7 @@ enum { GAR_SUM = 0, GAR_MAX = 1, GAR_MIN = 2 };
  *   gar_plan_status reports GAR_ETIMEOUT.  Same workspace and results as
  *   GAR_STEP_FAITHFUL. */
 enum { GAR_STEP_FAITHFUL = 0, GAR_FUSED = 1, GAR_STEP_PERSISTENT = 2 };
+#define GAR_FUSED_MAX_OPS 4096
 
 /* The permutation group T_P (Sec. "Communication description via permutations").
  * GAR_GROUP_CYCLIC: t_k(x) = x + k mod P (Table 1a), any P.

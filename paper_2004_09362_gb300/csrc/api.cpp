@@ -89,8 +89,23 @@ int prepare_step_faithful(gar_plan *pl) {
   return GAR_OK;
 }
 
+// Fused mode compiles the plan's program as straight-line code; the compile time grows
+// faster than linearly with its size (P = 300, 3900 operations: about a minute).
+int check_fused_size(const gar_plan *pl) {
+  const size_t ops = pl->prog.a.size() + 2 * (size_t)pl->P;
+  if (ops > GAR_FUSED_MAX_OPS) {
+    set_error("fused program of " + std::to_string(ops) + " operations (" +
+              std::to_string(pl->prog.a.size()) + " combines + " + std::to_string(2 * pl->P) +
+              " loads and stores) exceeds GAR_FUSED_MAX_OPS = " + std::to_string(GAR_FUSED_MAX_OPS) +
+              "; use GAR_STEP_FAITHFUL");
+    return GAR_EINVAL;
+  }
+  return GAR_OK;
+}
+
 int compile_fused(gar_plan *pl) {
   if (pl->fused) return GAR_OK;
+  if (int rc = check_fused_size(pl)) return rc;
   CodegenResult cg = generate_fused_source(*pl);
   JitKernel *k = nullptr;
   int rc = jit_compile(cg, &k);
@@ -596,6 +611,8 @@ int gar_allreduce_batched(gar_plan *const *plans, int nplans, const gar_batch_de
     ps.push_back(plans[k]);
   }
   if (count == 0 || plans[0]->n == 0) return GAR_OK;
+  for (const gar_plan *pl : ps)
+    if (int rc = check_fused_size(pl)) return rc;
   if (reinterpret_cast<uintptr_t>(desc) % 8 != 0) {
     set_error("descriptor array is not 8-byte aligned");
     return GAR_EALIGN;

@@ -148,7 +148,10 @@ struct LaunchView {
 };
 
 // Chunked mapping: work item `item` = (chunk, rank x, op) is done by the whole CTA.
-template <typename T, int OP, int MAXP>
+// kCopyPaths: copy-only ops take the deeper copy loops.  The persistent kernel, which
+// keeps its launch loop's state live around this body, leaves them out: with them it
+// needs 109 registers (2 CTAs per SM) instead of about 75 (3 CTAs per SM).
+template <typename T, int OP, int MAXP, bool kCopyPaths = true>
 __device__ __forceinline__ void chunk_work(const StepArgs<MAXP> &a, const LaunchView &lv, uint64_t item) {
   using A = typename AccOf<T>::type;
   const int chunk = (int)(item % (uint64_t)lv.nchunks);
@@ -242,7 +245,7 @@ __device__ __forceinline__ void chunk_work(const StepArgs<MAXP> &a, const Launch
       if (e < vend) store4<T, A>(op.out0_buf, out0, e, v[u]);
     }
   };
-  const bool copy_only = !out1 && (has_recv != (own0 != nullptr));
+  const bool copy_only = kCopyPaths && !out1 && (has_recv != (own0 != nullptr));
   const uint8_t copy_src_buf = has_recv ? op.recv_buf : op.out0_own;
   // A copy between buffers of one element type moves raw 4-element units (16 B, or 8 B
   // for bf16) with a compile-time stride: few registers, so 6 units per thread in flight
@@ -461,7 +464,8 @@ __global__ void __launch_bounds__(kThreads) step_kernel_persistent(const __grid_
                              (uint64_t)gridDim.x * blockDim.x);
     } else {
       const uint64_t items = (uint64_t)lv.nchunks * (uint64_t)p.s.P * (uint64_t)lv.nops;
-      for (uint64_t item = blockIdx.x; item < items; item += gridDim.x) chunk_work<T, OP, MAXP>(p.s, lv, item);
+      for (uint64_t item = blockIdx.x; item < items; item += gridDim.x)
+        chunk_work<T, OP, MAXP, false>(p.s, lv, item);
     }
     if (l + 1 < p.nlaunch && !grid_barrier(p.bar, expected, p.spin_limit, l)) return;
   }

@@ -23,6 +23,7 @@ GAR_STEPS_BO, GAR_STEPS_LO, GAR_STEPS_RING = -1, -2, -3
 GAR_GROUP_CYCLIC, GAR_GROUP_XOR = 0, 1
 GROUPS = {"cyclic": GAR_GROUP_CYCLIC, "xor": GAR_GROUP_XOR}
 GAR_MAX_P = 1024
+GAR_FUSED_MAX_OPS = 4096
 GAR_OK = 0
 
 DTYPES = {"f32": GAR_F32, "bf16": GAR_BF16, "i32": GAR_I32}

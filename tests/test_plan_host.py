@@ -34,6 +34,10 @@ def test_library_exports_every_declared_function():
     lib = ctypes.CDLL(gar.lib_path())
     for name in declared:
         assert hasattr(lib, name), name
+    # the binding's copies of the header's limits
+    for name in ("GAR_MAX_P", "GAR_FUSED_MAX_OPS"):
+        m = re.search(r"#define\s+" + name + r"\s+(\d+)", hdr)
+        assert m and int(m.group(1)) == getattr(gar, name), name
 
 
 def test_jit_compiles_without_gpu():
@@ -270,6 +274,24 @@ def test_fold_argument_errors():
     with pytest.raises(gar.GarError):
         gar.gar_plan_create_group(16, 10, steps=10, group="xor")
     assert gar.gar_plan_create(24, 10, steps=46).info()["S"] == 46
+
+
+def test_fused_program_size_limit():
+    """Fused mode compiles the program as straight-line code and refuses programs over
+    GAR_FUSED_MAX_OPS operations (combines + P loads + P stores) at once, with the sizes
+    in the message; the step-faithful mode still takes the plan."""
+    for (P, S) in [(1024, 10), (1024, 11), (512, 9)]:
+        plan = gar.gar_plan_create(P, 5000, "f32", "sum", S)
+        ops = plan.info()["fused_combines"] + 2 * P
+        assert ops > gar.GAR_FUSED_MAX_OPS
+        with pytest.raises(gar.GarError) as e:
+            gar.gar_plan_compile(plan, "fused")
+        assert e.value.code == -1
+        assert f"fused program of {ops} operations" in str(e.value)
+        gar.gar_plan_compile(plan, "step")
+    # the bandwidth-optimal program at the largest P is within the limit
+    plan = gar.gar_plan_create(gar.GAR_MAX_P, 5000, "f32", "sum", gar.GAR_STEPS_BO)
+    assert plan.info()["fused_combines"] + 2 * gar.GAR_MAX_P <= gar.GAR_FUSED_MAX_OPS
 
 
 def test_workspace_sizes():
