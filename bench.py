@@ -469,6 +469,9 @@ def measure_rows(gar, gar_inputs, stream, hbm_peak):
             ms_s = _time_loop(lambda: gar.gar_allreduce(plan, inp, "step", stream), 2, 1, stream)
             ent["step_ms"] = round(ms_s, 3)
             ent["step_launches"] = plan.info()["n_launches"]
+            dram = _step_dram_bytes(gar, plan, P, n, "bf16")
+            ent["step_dram_model_bytes"] = dram
+            ent["step_frac_dram_model"] = round(dram / ms_s / 1e6 / hbm_peak, 4)
             plan.workspace = None
             gar.gar_plan_set_workspace(plan, 0, 0)
         sweep[f"S{S}"] = ent

@@ -99,13 +99,13 @@ def test_mid_size_chunked_step_kernel(P):
     """Blocks of ~5000 elements with ragged starts: the chunked step-faithful launch
     (several chunks per block, 16-byte head/tail handling), every step count and type."""
     n = P * 5003 + 5
-    for dtype in ("f32", "i32", "bf16"):
+    for (dtype, op) in (("f32", "sum"), ("i32", "sum"), ("bf16", "sum"), ("bf16", "max")):
         t = _np_inputs(P, n, dtype, seed=33 * P)
         host = _to_host_list(t, dtype)
         for S in _Ss(P):
-            plan = gar.gar_plan_create(P, n, dtype, "sum", S)
-            _assert_same(_run(plan, t, "step"), G.allreduce(host, S, "sum", dtype), dtype,
-                         f"P={P} {dtype} S={S}")
+            plan = gar.gar_plan_create(P, n, dtype, op, S)
+            _assert_same(_run(plan, t, "step"), G.allreduce(host, S, op, dtype), dtype,
+                         f"P={P} {dtype} {op} S={S}")
             rec = gar.gar_last_step_bytes(plan)
             assert rec == gar.gar_plan_bytes(plan)[1]
 
