@@ -7,7 +7,8 @@
 // partner rank's block; the read value is combined in registers with the own block
 // (eq. distr_vectors_combination) and stored.  Every CTA owns one chunk of one block
 // of one (op, rank) pair.  Each warp counts the elements it read from partners and adds
-// the bytes to the step's counter, so the bytes a step actually moved are recorded.
+// the bytes to one of the step's counter slots, so the bytes a step actually moved are
+// recorded.
 #include <cuda_bf16.h>
 #include <cuda_runtime.h>
 
@@ -408,17 +409,46 @@ __device__ __forceinline__ LaunchView view_of(const StepArgs<MAXP> &a) {
   return lv;
 }
 
-template <typename T, int OP, int MAXP>
+// Programmatic dependent launch: the step launches of one Allreduce are made with
+// programmatic stream serialisation, so launch i+1's CTAs may become resident while
+// launch i drains.  griddepcontrol.wait blocks until every prerequisite grid has
+// completed and its memory is visible (a no-op without such a dependency); nothing is
+// read before it.  launch_dependents, issued once a CTA's work is done, lets the next
+// launch start once every CTA of this one has issued it or exited.
+__device__ __forceinline__ void wait_prior_grid() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
+__device__ __forceinline__ void allow_next_grid() { asm volatile("griddepcontrol.launch_dependents;" ::: "memory"); }
+
 // At most 40 registers (6 CTAs per SM): the bf16 launches ran 5-8 % faster than at the
 // 48 registers the compiler picks unbounded, fp32 the same.
+template <typename T, int OP, int MAXP>
 __global__ void __launch_bounds__(kThreads, 6) step_kernel(const __grid_constant__ StepArgs<MAXP> a) {
+  wait_prior_grid();
   chunk_work<T, OP, MAXP>(a, view_of(a), blockIdx.x);
+  allow_next_grid();
 }
 
 template <typename T, int OP, int MAXP>
 __global__ void __launch_bounds__(kThreads) step_kernel_flat(const __grid_constant__ StepArgs<MAXP> a) {
+  wait_prior_grid();
   flat_work<T, OP, MAXP>(a, view_of(a), (uint64_t)blockIdx.x * blockDim.x + threadIdx.x,
                          (uint64_t)gridDim.x * blockDim.x);
+  allow_next_grid();
+}
+
+// Launches a step kernel with programmatic stream serialisation (see above).
+template <typename Args>
+cudaError_t launch_pdl(void (*kernel)(Args), unsigned grid, gar_stream_t stream, const Args &a) {
+  cudaLaunchConfig_t cfg{};
+  cfg.gridDim = dim3(grid);
+  cfg.blockDim = dim3(kThreads);
+  cfg.dynamicSmemBytes = 0;
+  cfg.stream = (cudaStream_t)stream;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  return cudaLaunchKernelEx(&cfg, kernel, a);
 }
 
 // ---------------------------------------------------------------------------
@@ -565,8 +595,7 @@ int launch_typed(const gar_plan &pl, const Launch &ln, int launch_index, void *c
     const uint64_t total = (uint64_t)ln.nops * pl.n;
     const uint64_t grid = std::min<uint64_t>((total + kThreads - 1) / kThreads,
                                              (uint64_t)num_sms() * 32);
-    step_kernel_flat<T, OP, MAXP><<<(unsigned)grid, kThreads, 0, (cudaStream_t)stream>>>(a);
-    cudaError_t e = cudaGetLastError();
+    cudaError_t e = launch_pdl(step_kernel_flat<T, OP, MAXP>, (unsigned)grid, stream, a);
     if (e != cudaSuccess) return cuda_fail(e, "step kernel launch");
     return GAR_OK;
   }
@@ -580,8 +609,7 @@ int launch_typed(const gar_plan &pl, const Launch &ln, int launch_index, void *c
     set_error("step launch grid too large");
     return GAR_EINVAL;
   }
-  step_kernel<T, OP, MAXP><<<(unsigned)grid, kThreads, 0, (cudaStream_t)stream>>>(a);
-  cudaError_t e = cudaGetLastError();
+  cudaError_t e = launch_pdl(step_kernel<T, OP, MAXP>, (unsigned)grid, stream, a);
   if (e != cudaSuccess) return cuda_fail(e, "step kernel launch");
   return GAR_OK;
 }
