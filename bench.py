@@ -364,6 +364,7 @@ def run_ours(args):
         out["rows"] = measure_rows(gar, gar_inputs, stream, hbm_peak)
     if rank == 0 and not args.no_cpu:
         out["cpu_baseline"] = cpu_baseline_sample(target_s=args.cpu_seconds)
+        out["cpu_baseline_mt"] = cpu_column_baseline()
     if dist is not None:
         dist.barrier()
         dist.destroy_process_group()
@@ -696,6 +697,32 @@ def cpu_baseline_sample(target_s=10.0):
             "cpu_model": model, "kind": "oracle", "seconds": round(total, 2),
             "sample": f"P=24, S=10 (bandwidth-optimal), fp32 sum, n={n} elements per rank "
                       f"(headline has {n_max}), {reps} Allreduce(s), mean time"}
+
+
+def cpu_column_baseline(target_s=3.0):
+    """The plain multi-threaded CPU Allreduce (oracle/column_reduce.c: rank-order column
+    reduction written to every rank, one thread per host core) on the full headline
+    shape, P = 24 x 16,777,216 fp32, repeated for about target_s seconds.  A second,
+    stronger CPU baseline beside the single-threaded oracle; same unit."""
+    import numpy as np
+    from oracle import column_reduce as CR
+    P, n = 24, 16777216
+    rng = np.random.default_rng(0)
+    xs = [(rng.standard_normal(n) * 1e-3).astype(np.float32) for _ in range(P)]
+    outs = [np.empty(n, np.float32) for _ in range(P)]
+    ip, op_ = [v.ctypes.data for v in xs], [o.ctypes.data for o in outs]
+    cores, model = _cpu_info()
+    CR.column_allreduce_ptrs(ip, op_, n, "f32", "sum", cores)      # warm-up (first touch)
+    reps, total = 0, 0.0
+    while total < target_s or reps < 3:
+        t0 = time.perf_counter()
+        CR.column_allreduce_ptrs(ip, op_, n, "f32", "sum", cores)
+        total += time.perf_counter() - t0
+        reps += 1
+    sec = total / reps
+    return {"value": round(_alg_bytes(P, n, "f32") / sec / 1e9, 3), "unit": "GB/s",
+            "cores": cores, "cpu_model": model, "kind": "plain column reduction (C, pthreads)",
+            "sample": f"P=24 x n=16777216 fp32 sum (the headline shape), {reps} runs, mean time"}
 
 
 def run_reference(args):

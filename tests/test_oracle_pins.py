@@ -719,3 +719,54 @@ def test_fold_schedule_ends():
         G.simulate(8, 0, 9)                      # odd S beyond 2L
     with pytest.raises(ValueError):
         G.simulate(8, 0, 16)                     # beyond 2(P-1)
+
+
+# ---------------------------------------------------------------------------
+# A second implementation of the definition (oracle/column_reduce.c)
+# ---------------------------------------------------------------------------
+
+@pytest.mark.parametrize("threads", [1, 3])
+def test_column_reduce_is_the_definition(threads):
+    """The C column reduction against numpy's column reduction: int32 wraparound sums
+    and max/min exactly, fp32 sums within the rank-order rounding of a float64 sum."""
+    from oracle import column_reduce as CR
+    rng = np.random.default_rng(11)
+    P, n = 7, 1001
+    xi = [rng.integers(-2 ** 31, 2 ** 31, n, dtype=np.int64).astype(np.int32) for _ in range(P)]
+    want = np.zeros(n, np.int64)
+    for v in xi:
+        want += v
+    want = ((want + 2 ** 31) % 2 ** 32 - 2 ** 31).astype(np.int32)
+    for o in CR.column_allreduce(xi, "sum", "i32", threads):
+        np.testing.assert_array_equal(o, want)
+    for op, f in (("max", np.max), ("min", np.min)):
+        for dt, xs in (("i32", xi), ("f32", [v.astype(np.float32) for v in xi])):
+            for o in CR.column_allreduce(xs, op, dt, threads):
+                np.testing.assert_array_equal(o, f(np.stack(xs), axis=0))
+    xf = [rng.standard_normal(n).astype(np.float32) for _ in range(P)]
+    exact = np.sum(np.stack(xf).astype(np.float64), axis=0)
+    for o in CR.column_allreduce(xf, "sum", "f32", threads):
+        np.testing.assert_array_equal(o, exact.astype(np.float32))
+
+
+@pytest.mark.parametrize("P", [2, 3, 5, 7, 8, 12, 24, 33])
+def test_oracle_order_free_results_equal_column_reduce(P):
+    """Where the result does not depend on the association order (int32 wraparound sum,
+    max, min), every schedule of the oracle -- every S, both groups, folds, the Ring --
+    equals the plain column reduction bit for bit."""
+    from oracle import column_reduce as CR
+    rng = np.random.default_rng(100 + P)
+    n = 3 * P + 2
+    xi = [rng.integers(-2 ** 31, 2 ** 31, n, dtype=np.int64).astype(np.int32) for _ in range(P)]
+    xf = [rng.standard_normal(n).astype(np.float32) for _ in range(P)]
+    L = G.ceil_log2(P)
+    sched = [(S, "cyclic") for S in range(L, 2 * L + 1)]
+    sched += [(S, "cyclic") for S in range(2 * L + 2, 2 * (P - 1) + 1, 2)]
+    if P & (P - 1) == 0:
+        sched += [(S, "xor") for S in range(L, 2 * L + 1)]
+    for (S, group) in sched + [("ring", "cyclic")]:
+        for (dt, xs, op) in (("i32", xi, "sum"), ("i32", xi, "max"), ("f32", xf, "min")):
+            want = CR.column_allreduce(xs, op, dt)[0]
+            for o in G.allreduce(xs, S, op, dt, group=group):
+                np.testing.assert_array_equal(o, want, err_msg=f"P={P} S={S} {group} {dt} {op}")
+
