@@ -2,11 +2,13 @@
  * gar.h -- permutation-group Allreduce on one GB300 (sm_103a).
  *
  * Implements the generalized Allreduce of D. Kolmakov and X. Zhang, "A Generalization
- * of the Allreduce Operation" (arXiv 2004.09362): the schedule built from the cyclic
- * permutation group T_P, with a step count S that can be set anywhere from
- * ceil(log2 P) (latency-optimal, Sec. "Latency-optimal version") to 2 ceil(log2 P)
- * (bandwidth-optimal, Sec. "Bandwidth-optimal algorithm") for any P, including
- * non-powers of two and primes (Sec. "Moving towards latency-optimal version").
+ * of the Allreduce Operation" (arXiv 2004.09362): the schedule built from a
+ * permutation group T_P (the cyclic group for any P, including non-powers of two and
+ * primes; the XOR group of Table 1b for powers of two), with a step count S that can be
+ * set anywhere from ceil(log2 P) (latency-optimal, Sec. "Latency-optimal version") to
+ * 2 ceil(log2 P) (bandwidth-optimal, Sec. "Bandwidth-optimal algorithm"; between them
+ * Sec. "Moving towards latency-optimal version"), and beyond that up to the Ring's
+ * 2(P-1) steps (fold schedules, GAR_STEPS_RING).
  *
  * The P processes of the paper are P "virtual ranks": P equally sized vectors that
  * all live in the memory of one GPU.  A message of the paper is a read of the partner
@@ -58,7 +60,9 @@ enum { GAR_SUM = 0, GAR_MAX = 1, GAR_MIN = 2 };
  * GAR_STEP_FAITHFUL: one kernel launch per schedule step; a step reads the
  *   partner rank's blocks (the paper's send/receive) with 16-byte vector loads and
  *   combines them with the own block; needs the workspace reported by
- *   gar_plan_bytes; records the bytes read from partners per step.
+ *   gar_plan_bytes; records the bytes read from partners per step.  The launches of
+ *   one call are chained by programmatic dependent launch: a launch may become resident
+ *   early but reads nothing before every earlier kernel on the stream has completed.
  * GAR_FUSED: one launch for the whole Allreduce; per element position the P
  *   contributions are loaded once, the reduction program that the schedule induces
  *   runs in registers, and every rank's result is written once.  The program becomes
@@ -108,7 +112,7 @@ enum {
 /* Describes a plan.  Symbols follow the paper: L = ceil(log2 P) reduction steps
  * (eq. bo_starting_set_size), S = 2L - r total steps, K = number of q_Sigma copies at
  * the end of the reduction phase (K = N_{L-r}; K = 1 bandwidth-optimal, K = P
- * latency-optimal). */
+ * latency-optimal).  Fold schedules and the Ring have S > 2L, r = 0 and K = 1. */
 typedef struct {
   int32_t P;
   int32_t L;
@@ -155,7 +159,7 @@ GAR_API void gar_plan_destroy(gar_plan *plan);
 GAR_API int gar_plan_get_info(const gar_plan *plan, gar_plan_info *info);
 
 /* Sizes.  workspace_bytes: device workspace step-faithful mode needs (0 when the
- * schedule runs in place: bandwidth-optimal f32/i32).  msg_bytes_per_step (may be
+ * schedule runs in place: bandwidth-optimal, fold and Ring schedules in f32/i32).  msg_bytes_per_step (may be
  * NULL, else S entries): bytes all ranks together read from their partners in each
  * communication step, the schedule's message volume (Sec. "Communication
  * operator": every rank sends its blocks of the transmitted vectors).  S (may be
@@ -166,7 +170,8 @@ GAR_API int gar_plan_bytes(const gar_plan *plan, size_t *workspace_bytes,
 /* Schedule introspection (host-only).  For communication step t in [0, S):
  * phase = 0 (reduction) or 1 (distribution); partner: rank x receives from rank
  * (x + partner) mod P in the cyclic group (reduction: +floor(N_i/2), eq. bo_dir_perms;
- * distribution: -floor(N_i/2); the Ring: -1 in both phases) and from rank x XOR
+ * distribution: -floor(N_i/2); fold schedules: +f_i and -f_i, f_i the vectors folded
+ * in reduction step i; the Ring: -1 in both phases) and from rank x XOR
  * partner in the XOR group; placements[0..*count) = placements of the vectors each rank
  * transmits (eq. bo_tx_dist and its shifted forms).  placements may be NULL to query
  * the count; otherwise it must hold P entries. */
@@ -214,10 +219,11 @@ GAR_API int gar_plan_prepare(gar_plan *plan, int mode);
  * rank_buffers: host array of P device pointers, each to n elements of the plan's
  * type, 16-byte aligned and pairwise distinct.  On return the work is enqueued on
  * `stream`; when it completes every buffer holds the reduction.  Rank x's block b is
- * the value at placement (x - b) mod P after the paper's schedule; for bandwidth-
- * optimal plans all ranks get identical bits, otherwise floating-point sums may differ
- * in the last bits between ranks (each rank's association order is a rotation of the
- * same tree). */
+ * the value at placement (x - b) mod P (x XOR b in the XOR group) after the paper's
+ * schedule; for plans with one result copy (K = 1: bandwidth-optimal, fold and Ring
+ * schedules) all ranks get identical bits, otherwise floating-point sums may differ in
+ * the last bits between ranks (each rank's association order is a rotation of the same
+ * tree).  The modes give identical bits. */
 GAR_API int gar_allreduce(gar_plan *plan, void *const *rank_buffers, int mode, gar_stream_t stream);
 
 /* Host-buffer Allreduce: the P inputs host_in[x] are in host memory and the P results
