@@ -166,6 +166,23 @@ int grid_for(const JitKernel *k, uint64_t work_items) {
   return (int)std::max<uint64_t>(1, std::min<uint64_t>(need, cap));
 }
 
+// Launches a generated kernel with programmatic stream serialisation: back-to-back
+// calls overlap one launch's start with the previous one's drain.  Every generated
+// kernel runs griddepcontrol.wait before its first read, so it still sees all the work
+// of earlier kernels on the stream.
+cudaError_t launch_generated(const JitKernel *k, int grid, void **kargs, gar_stream_t stream) {
+  cudaLaunchConfig_t cfg{};
+  cfg.gridDim = dim3(grid);
+  cfg.blockDim = dim3(k->threads);
+  cfg.stream = (cudaStream_t)stream;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  return cudaLaunchKernelExC(&cfg, (const void *)k->kernel, kargs);
+}
+
 // One fused launch over element positions [e_lo, e_hi) (e_lo a multiple of the
 // kernel's vector width).  The parameter block is the generated kernel's gar_args:
 // P input pointers, P output pointers, e_lo, e_hi.
@@ -181,8 +198,7 @@ int launch_fused_range(gar_plan *pl, const void *const *in, void *const *out, ui
   void *kargs[] = {args.data()};
   const uint64_t items = (e_hi - e_lo) / pl->fused->width + 1;
   const int grid = grid_for(pl->fused, items);
-  cudaError_t e = cudaLaunchKernel((const void *)pl->fused->kernel, dim3(grid),
-                                   dim3(pl->fused->threads), kargs, 0, (cudaStream_t)stream);
+  cudaError_t e = launch_generated(pl->fused, grid, kargs, stream);
   if (e != cudaSuccess) return cuda_fail(e, "fused kernel launch");
   return GAR_OK;
 }
@@ -630,8 +646,7 @@ int gar_allreduce_batched(gar_plan *const *plans, int nplans, const gar_batch_de
   void *kargs[] = {&a};
   const uint64_t per = plans[0]->n / k->width + plans[0]->n % k->width;
   const int grid = grid_for(k, per * (uint64_t)count);
-  cudaError_t e = cudaLaunchKernel((const void *)k->kernel, dim3(grid), dim3(k->threads), kargs, 0,
-                                   (cudaStream_t)stream);
+  cudaError_t e = launch_generated(k, grid, kargs, stream);
   if (e != cudaSuccess) return cuda_fail(e, "batched kernel launch");
   return GAR_OK;
 }

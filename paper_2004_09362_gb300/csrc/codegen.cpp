@@ -346,6 +346,9 @@ CodegenResult generate_fused_source(const gar_plan &pl) {
                  pl.group == GAR_GROUP_XOR);
   s += "extern \"C\" __global__ void " + bounds + " " + cg.kernel_name +
        "(const __grid_constant__ gar_args a) {\n";
+  // launched with programmatic stream serialisation: nothing is read before every
+  // earlier kernel on the stream has completed
+  s += "  asm volatile(\"griddepcontrol.wait;\" ::: \"memory\");\n";
   s += "  const gar_u64 v_lo = a.e_lo / GAR_W, v_hi = a.e_hi / GAR_W;\n";
   s += "  const gar_u64 stride = (gar_u64)gridDim.x * blockDim.x;\n";
   s += "  const gar_u64 tid = (gar_u64)blockIdx.x * blockDim.x + threadIdx.x;\n";
@@ -366,7 +369,8 @@ CodegenResult generate_fused_source(const gar_plan &pl) {
   s += "  if (tid < a.e_hi - t0) {\n";
   s += "    const gar_u64 e = t0 + tid;\n";
   s += rotate ? "    gar_eval_plan<1>(a, e, gar_block_of(e));\n" : "    gar_eval_plan<1>(a, e, 0);\n";
-  s += "  }\n}\n";
+  s += "  }\n";
+  s += "  asm volatile(\"griddepcontrol.launch_dependents;\" ::: \"memory\");\n}\n";
   cg.source = s;
   return cg;
 }
@@ -418,6 +422,9 @@ CodegenResult generate_batched_source(const std::vector<const gar_plan *> &plans
   // with fewer threads than items the descriptor latency overlaps the data loads.
   s += "  gar_u64 g = (gar_u64)blockIdx.x * blockDim.x + threadIdx.x;\n";
   s += "  if (g >= total) return;\n";
+  // launched with programmatic stream serialisation: nothing is read before every
+  // earlier kernel on the stream has completed
+  s += "  asm volatile(\"griddepcontrol.wait;\" ::: \"memory\");\n";
   s += "  gar_desc dn = a.desc[g / per];\n";
   s += "  for (; g < total; g += stride) {\n";
   s += "    const gar_u64 i = g / per, v = g - i * per;\n";
@@ -451,7 +458,8 @@ CodegenResult generate_batched_source(const std::vector<const gar_plan *> &plans
                 : "        gar_eval_" + tag + "<1>(in, out, e, 0);\n";
     s += "      }\n      break;\n";
   }
-  s += "    default: break;\n    }\n  }\n}\n";
+  s += "    default: break;\n    }\n  }\n";
+  s += "  asm volatile(\"griddepcontrol.launch_dependents;\" ::: \"memory\");\n}\n";
   cg.source = s;
   return cg;
 }
