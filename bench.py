@@ -459,7 +459,10 @@ def measure_rows(gar, gar_inputs, stream, hbm_peak):
     for S in wl.steps:
         plan = gar.gar_plan_create(P, n, "bf16", "sum", S)
         gar.gar_plan_prepare(plan, "fused")
-        ms_f = _time_loop(lambda: gar.gar_allreduce(plan, inp, "fused", stream), 5, 3, stream)
+        # median of 5 loops of 10 launches (single short loops varied by up to 5 %)
+        ms_f = statistics.median(
+            _time_loop(lambda: gar.gar_allreduce(plan, inp, "fused", stream), 10, 3 if k == 0 else 1,
+                       stream) for k in range(5))
         ent = {"fused_ms": round(ms_f, 4),
                "fused_GB/s": round(_alg_bytes(P, n, "bf16") / ms_f / 1e6, 1),
                "fused_frac": round(_alg_bytes(P, n, "bf16") / ms_f / 1e6 / hbm_peak, 4),

@@ -189,12 +189,16 @@ cudaError_t launch_generated(const JitKernel *k, int grid, void **kargs, gar_str
 int launch_fused_range(gar_plan *pl, const void *const *in, void *const *out, uint64_t e_lo,
                        uint64_t e_hi, gar_stream_t stream) {
   if (e_hi <= e_lo) return GAR_OK;
+  // gar_args: the in[] table, then the out[] table, each table_copies times in a row,
+  // then e_lo, e_hi
   const size_t pb = 8 * (size_t)pl->P;
-  std::vector<unsigned char> args(2 * pb + 16);
-  std::memcpy(args.data(), in, pb);
-  std::memcpy(args.data() + pb, out, pb);
-  std::memcpy(args.data() + 2 * pb, &e_lo, 8);
-  std::memcpy(args.data() + 2 * pb + 8, &e_hi, 8);
+  const int copies = pl->fused->table_copies;
+  std::vector<unsigned char> args(2 * copies * pb + 16);
+  unsigned char *w = args.data();
+  for (int c = 0; c < copies; ++c, w += pb) std::memcpy(w, in, pb);
+  for (int c = 0; c < copies; ++c, w += pb) std::memcpy(w, out, pb);
+  std::memcpy(w, &e_lo, 8);
+  std::memcpy(w + 8, &e_hi, 8);
   void *kargs[] = {args.data()};
   const uint64_t items = (e_hi - e_lo) / pl->fused->width + 1;
   const int grid = grid_for(pl->fused, items);

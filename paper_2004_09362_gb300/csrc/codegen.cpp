@@ -255,7 +255,7 @@ std::string emit_eval(const FusedProgram &fp, const Schedule &sc, const std::str
                       const std::string &params,
                       const std::function<std::string(const std::string &)> &ld_row,
                       const std::function<std::string(const std::string &)> &st_row,
-                      bool rotate, bool xor_group) {
+                      bool rotate, bool xor_group, bool doubled = false) {
   const int P = fp.P;
   std::string s;
   s += "template <int W>\nstatic __device__ __forceinline__ void gar_eval_" + tag + "(" + params +
@@ -266,6 +266,8 @@ std::string emit_eval(const FusedProgram &fp, const Schedule &sc, const std::str
     if (!rotate) return std::to_string(j);
     if (j == 0) return "b";
     if (xor_group) return fmt("(b ^ %d)", j);
+    // with the pointer tables stored twice, entry b + j (< 2P) is rank (b + j) mod P
+    if (doubled) return fmt("(b + %d)", j);
     return fmt("(b + %d >= %d ? b + %d : b + %d)", j, P, j - P, j);
   };
   // stores of result s go to every placement p whose origin is s
@@ -338,12 +340,21 @@ CodegenResult generate_fused_source(const gar_plan &pl) {
   // in[] / out[]: where rank x's contributions are read and its results written (equal
   // for the in-place Allreduce); [e_lo, e_hi): the element positions this launch covers
   // (e_lo a multiple of GAR_W), so one Allreduce can run as several launches.
-  s += fmt("struct gar_args { const gar_io *in[%d]; gar_io *out[%d]; gar_u64 e_lo, e_hi; };\n", P, P);
+  // Rotated cyclic programs index the pointer tables with (b + j) mod P; storing each
+  // table twice turns that into b + j, which folds into the constant-bank offset of the
+  // pointer load (the parameter block stays within 32 KB up to P = 1000).  Only for
+  // programs with several result copies (K > 1): there it freed registers and made P = 127
+  // bf16 up to 19 % faster (S = 8..13); the single-copy programs (bandwidth-optimal, folds,
+  // the Ring) are HBM-bound and ran 0.6-0.8 % slower with it.
+  const bool doubled = rotate && pl.group != GAR_GROUP_XOR && P <= 1000 && pl.K > 1;
+  cg.table_copies = doubled ? 2 : 1;
+  s += fmt("struct gar_args { const gar_io *in[%d]; gar_io *out[%d]; gar_u64 e_lo, e_hi; };\n",
+           cg.table_copies * P, cg.table_copies * P);
   s += emit_block_of("gar_block_of", P, pl.n);
   auto ld_row = [](const std::string &r) { return "a.in[" + r + "]"; };
   auto st_row = [](const std::string &r) { return "a.out[" + r + "]"; };
   s += emit_eval(fp, sc, "plan", "const gar_args &a", ld_row, st_row, rotate,
-                 pl.group == GAR_GROUP_XOR);
+                 pl.group == GAR_GROUP_XOR, doubled);
   s += "extern \"C\" __global__ void " + bounds + " " + cg.kernel_name +
        "(const __grid_constant__ gar_args a) {\n";
   // launched with programmatic stream serialisation: nothing is read before every

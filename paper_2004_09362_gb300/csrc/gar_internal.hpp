@@ -131,6 +131,7 @@ struct CodegenResult {
   std::string source;
   std::string kernel_name;
   int width = 1;
+  int table_copies = 1;  // fused kernels: copies of the in[] / out[] pointer tables (1 or 2)
 };
 CodegenResult generate_fused_source(const gar_plan &pl);
 CodegenResult generate_batched_source(const std::vector<const gar_plan *> &plans);
@@ -142,6 +143,7 @@ struct JitKernel {
   std::vector<char> cubin;
   std::string name;
   int width = 1;
+  int table_copies = 1;
   int threads = 256;
   int blocks_per_sm = 0;
   int regs = 0, local_bytes = 0;

@@ -58,6 +58,7 @@ int jit_compile(const CodegenResult &cg, JitKernel **out) {
   nvrtcDestroyProgram(&prog);
   k->name = cg.kernel_name;
   k->width = cg.width;
+  k->table_copies = cg.table_copies;
   *out = k.get();
   g_cache.emplace(cg.source, std::move(k));
   return GAR_OK;

@@ -28,11 +28,13 @@ def _padded(t):
 
 
 @pytest.mark.parametrize("S,mode", [(10, "step"), (15, "step"), (20, "step"), (20, "fused"),
-                                    (20, "persistent")])
+                                    (19, "fused"), (20, "persistent")])
 def test_maximum_p(S, mode):
     """P = 1024 ranks, 3 or 4 elements per block: step-faithful at the latency-optimal,
-    an intermediate and the bandwidth-optimal step count; fused and persistent at the
-    bandwidth-optimal one (the latency-optimal fused program exceeds GAR_FUSED_MAX_OPS)."""
+    an intermediate and the bandwidth-optimal step count; fused at the bandwidth-optimal
+    one and at S = 19 (K = 2: a rotated program whose pointer tables are too large to
+    store twice); persistent at the bandwidth-optimal one.  The latency-optimal fused
+    program exceeds GAR_FUSED_MAX_OPS."""
     P = gar.GAR_MAX_P
     n = 3 * P + 5
     t = gar_inputs.rank_inputs(P, n, "f32", ("normal", 0.0, 1.0), 1024 + S)
