@@ -316,7 +316,11 @@ CodegenResult generate_fused_source(const gar_plan &pl) {
   const FusedProgram &fp = pl.prog;
   const int P = pl.P;
   Schedule sc = order_program(fp);
-  int W = choose_width(pl.dtype, sc.peak_live, 16);
+  const bool rotate = pl.K != P;   // latency-optimal results do not depend on the block
+  const bool doubled = rotate && pl.group != GAR_GROUP_XOR && P <= 1000 && pl.K > 1;
+  // bf16 programs with doubled pointer tables (below) run best with at most 8-byte
+  // vectors (P = 127, S = 8..13: W = 8 was 3-6 % slower at S = 12, 13 than W = 4).
+  int W = choose_width(pl.dtype, sc.peak_live, (doubled && pl.dtype == GAR_BF16) ? 4 : 16);
   // Few element positions: narrower vectors give more threads, and the contributions'
   // load latencies then overlap across warps instead of queueing in one (P = 127 bf16
   // with 212 positions: 92 us at W = 8, 24 us at W = 1).
@@ -325,7 +329,6 @@ CodegenResult generate_fused_source(const gar_plan &pl) {
     if (w > 0 && (w & (w - 1)) == 0 && w * elem_size(pl.dtype) <= 16) W = w;
   const int minb = tune_int("GAR_TUNE_FUSED_MINB", 0);
   const std::string bounds = minb > 0 ? fmt("__launch_bounds__(256, %d)", minb) : "__launch_bounds__(256)";
-  const bool rotate = pl.K != P;   // latency-optimal results do not depend on the block
   CodegenResult cg;
   cg.width = W;
   cg.kernel_name = fmt("gar_fused_P%d_S%d_K%d_", P, pl.S, pl.K) + dtype_tag(pl.dtype) + "_" +
@@ -346,7 +349,6 @@ CodegenResult generate_fused_source(const gar_plan &pl) {
   // programs with several result copies (K > 1): there it freed registers and made P = 127
   // bf16 up to 19 % faster (S = 8..13); the single-copy programs (bandwidth-optimal, folds,
   // the Ring) are HBM-bound and ran 0.6-0.8 % slower with it.
-  const bool doubled = rotate && pl.group != GAR_GROUP_XOR && P <= 1000 && pl.K > 1;
   cg.table_copies = doubled ? 2 : 1;
   s += fmt("struct gar_args { const gar_io *in[%d]; gar_io *out[%d]; gar_u64 e_lo, e_hi; };\n",
            cg.table_copies * P, cg.table_copies * P);
