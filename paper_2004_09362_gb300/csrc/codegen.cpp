@@ -353,12 +353,26 @@ CodegenResult generate_fused_source(const gar_plan &pl) {
   s += fmt("struct gar_args { const gar_io *in[%d]; gar_io *out[%d]; gar_u64 e_lo, e_hi; };\n",
            cg.table_copies * P, cg.table_copies * P);
   s += emit_block_of("gar_block_of", P, pl.n);
-  auto ld_row = [](const std::string &r) { return "a.in[" + r + "]"; };
-  auto st_row = [](const std::string &r) { return "a.out[" + r + "]"; };
-  s += emit_eval(fp, sc, "plan", "const gar_args &a", ld_row, st_row, rotate,
-                 pl.group == GAR_GROUP_XOR, doubled);
+  // When blocks are shorter than a warp's span, the lanes of a warp work on different
+  // blocks b, and a rotated program's pointer index (b + j) differs across the warp:
+  // indexing the kernel parameters with it serialises (P = 127, 425 B: 34 us against
+  // 5.6 us unrotated).  Such kernels first copy the tables to shared memory, where
+  // divergent indices are cheap.
+  const int tp = cg.table_copies * P;
+  const bool staged = rotate && pl.n / (uint64_t)P < 32ull * (uint64_t)W;
+  auto ld_row = [staged](const std::string &r) { return (staged ? "tin[" : "a.in[") + r + "]"; };
+  auto st_row = [staged](const std::string &r) { return (staged ? "tout[" : "a.out[") + r + "]"; };
+  s += emit_eval(fp, sc, "plan",
+                 staged ? "const gar_io *const *tin, gar_io *const *tout" : "const gar_args &a", ld_row,
+                 st_row, rotate, pl.group == GAR_GROUP_XOR, doubled);
+  const std::string ev_args = staged ? "s_in, s_out" : "a";
   s += "extern \"C\" __global__ void " + bounds + " " + cg.kernel_name +
        "(const __grid_constant__ gar_args a) {\n";
+  if (staged) {
+    s += fmt("  __shared__ const gar_io *s_in[%d];\n  __shared__ gar_io *s_out[%d];\n", tp, tp);
+    s += fmt("  for (int i = threadIdx.x; i < %d; i += blockDim.x) { s_in[i] = a.in[i]; s_out[i] = a.out[i]; }\n", tp);
+    s += "  __syncthreads();\n";
+  }
   // launched with programmatic stream serialisation: nothing is read before every
   // earlier kernel on the stream has completed
   s += "  asm volatile(\"griddepcontrol.wait;\" ::: \"memory\");\n";
@@ -370,18 +384,19 @@ CodegenResult generate_fused_source(const gar_plan &pl) {
   if (rotate) {
     s += "    const int b0 = gar_block_of(e0);\n";
     s += "    if (GAR_W == 1 || b0 == gar_block_of(e0 + GAR_W - 1)) {\n";
-    s += "      gar_eval_plan<GAR_W>(a, e0, b0);\n";
+    s += "      gar_eval_plan<GAR_W>(" + ev_args + ", e0, b0);\n";
     s += "    } else {\n";
-    s += "      for (int w = 0; w < GAR_W; ++w) gar_eval_plan<1>(a, e0 + w, gar_block_of(e0 + w));\n";
+    s += "      for (int w = 0; w < GAR_W; ++w) gar_eval_plan<1>(" + ev_args + ", e0 + w, gar_block_of(e0 + w));\n";
     s += "    }\n";
   } else {
-    s += "    gar_eval_plan<GAR_W>(a, e0, 0);\n";
+    s += "    gar_eval_plan<GAR_W>(" + ev_args + ", e0, 0);\n";
   }
   s += "  }\n";
   s += "  const gar_u64 t0 = (v_hi * GAR_W > a.e_lo ? v_hi * GAR_W : a.e_lo);\n";
   s += "  if (tid < a.e_hi - t0) {\n";
   s += "    const gar_u64 e = t0 + tid;\n";
-  s += rotate ? "    gar_eval_plan<1>(a, e, gar_block_of(e));\n" : "    gar_eval_plan<1>(a, e, 0);\n";
+  s += rotate ? "    gar_eval_plan<1>(" + ev_args + ", e, gar_block_of(e));\n"
+              : "    gar_eval_plan<1>(" + ev_args + ", e, 0);\n";
   s += "  }\n";
   s += "  asm volatile(\"griddepcontrol.launch_dependents;\" ::: \"memory\");\n}\n";
   cg.source = s;

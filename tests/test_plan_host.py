@@ -294,6 +294,54 @@ def test_fused_program_size_limit():
     assert plan.info()["fused_combines"] + 2 * gar.GAR_MAX_P <= gar.GAR_FUSED_MAX_OPS
 
 
+@pytest.mark.parametrize("P,n,S", [(2, 1, 1), (3, 7, 2), (5, 1031, 3), (24, 5000, 5), (24, 1 << 20, 7),
+                                   (24, 1 << 20, 10), (127, 212, 7), (127, 212, 10), (127, 212, 14),
+                                   (1000, 5, 10)])
+def test_fused_parameter_layout(P, n, S):
+    """The generated kernel's gar_args must match the host packing in launch_fused_range:
+    in[c P], out[c P], e_lo, e_hi, with c = 2 (tables stored twice) exactly for rotated
+    programs with several result copies (1 < K < P), else 1; kernels whose warps span
+    several blocks copy the tables to shared memory of the same size."""
+    plan = gar.gar_plan_create(P, n, "f32", "sum", S)
+    src = gar.gar_plan_fused_source(plan)
+    m = re.search(r"struct gar_args \{ const gar_io \*in\[(\d+)\]; gar_io \*out\[(\d+)\]; "
+                  r"gar_u64 e_lo, e_hi; \};", src)
+    assert m, "unknown parameter layout"
+    c = int(m.group(1)) // P
+    assert int(m.group(1)) == int(m.group(2)) == c * P and c in (1, 2)
+    K = plan.info()["K"]
+    assert (c == 2) == (1 < K < P)
+    if "__shared__" in src:
+        assert K < P                          # only rotated programs are staged
+        assert f"__shared__ const gar_io *s_in[{c * P}];" in src
+
+
+@pytest.mark.parametrize("P", list(range(2, 41)) + [63, 64, 65, 127, 128])
+def test_result_copies_are_shifted_trees(P):
+    """Result copy s of the fused program is copy 0's tree with every leaf index shifted
+    by s (mod P): the K copies are one schedule shifted by s (cyclic group)."""
+    L = G.ceil_log2(P)
+    for S in range(L, 2 * L):
+        plan = gar.gar_plan_create(P, 1000, "f32", "sum", S)
+        pairs, outs = gar.gar_plan_fused_program(plan)
+        memo = {}
+
+        def tree(v):
+            if v < P:
+                return v
+            if v not in memo:
+                a, b = pairs[v - P]
+                memo[v] = (tree(a), tree(b))
+            return memo[v]
+
+        def shift(t, s):
+            return (t + s) % P if isinstance(t, int) else (shift(t[0], s), shift(t[1], s))
+
+        t0 = tree(outs[0])
+        for s in range(len(outs)):
+            assert tree(outs[s]) == shift(t0, s), (P, S, s)
+
+
 def test_workspace_sizes():
     # bandwidth-optimal fp32/int32 runs in place
     for P in (2, 5, 24, 127):
