@@ -266,11 +266,29 @@ def _stream_handle(stream) -> ctypes.c_void_p:
     return ctypes.c_void_p(int(stream) or None)
 
 
+def rank_pointer_array(rank_buffers) -> ctypes.Array:
+    """The P addresses as the C array of pointers the library's calls take: from a 2-D
+    tensor (rows = ranks), a list of tensors or ints, or an array this function returned
+    (passed through).  Build it once and pass it to every call to skip the per-call
+    marshalling (a few microseconds at P = 127)."""
+    if isinstance(rank_buffers, ctypes.Array):
+        return rank_buffers
+    if hasattr(rank_buffers, "dim") and rank_buffers.dim() == 2:
+        t = rank_buffers
+        if t.stride(1) != 1:
+            raise ValueError("rows must be contiguous")
+        a = (np.arange(t.shape[0], dtype=np.uint64) * np.uint64(t.stride(0) * t.element_size())
+             + np.uint64(t.data_ptr()))
+    elif len(rank_buffers) and isinstance(rank_buffers[0], int):
+        a = np.array(rank_buffers, dtype=np.uint64)
+    else:
+        a = np.array([int(b) if isinstance(b, int) else b.data_ptr() for b in rank_buffers],
+                     dtype=np.uint64)
+    return (ctypes.c_void_p * len(a)).from_buffer(a)    # keeps `a` alive
+
+
 def _ptr_array(ptrs) -> ctypes.Array:
-    arr = (ctypes.c_void_p * len(ptrs))()
-    for k, p in enumerate(ptrs):
-        arr[k] = int(p)
-    return arr
+    return rank_pointer_array(ptrs)
 
 
 def rank_pointers(rank_buffers) -> list[int]:
@@ -315,7 +333,7 @@ def gar_allreduce(plan: Plan, rank_buffers, mode="fused", stream=None) -> None:
     mode_c = _code(mode, MODES, "mode")
     if mode_c in (GAR_STEP_FAITHFUL, GAR_STEP_PERSISTENT) and plan.workspace is None:
         ensure_workspace(plan)
-    ptrs = _ptr_array(rank_pointers(rank_buffers))
+    ptrs = rank_pointer_array(rank_buffers)
     _check(_lib.gar_allreduce(plan.handle, ptrs, mode_c, _stream_handle(stream)), "gar_allreduce")
 
 
@@ -323,9 +341,9 @@ def gar_allreduce_host(plan: Plan, host_in, host_out, dev_bufs, mode="fused", st
     mode_c = _code(mode, MODES, "mode")
     if mode_c in (GAR_STEP_FAITHFUL, GAR_STEP_PERSISTENT) and plan.workspace is None:
         ensure_workspace(plan)
-    hin = _ptr_array(rank_pointers(host_in))
-    hout = _ptr_array(rank_pointers(host_out))
-    dev = _ptr_array(rank_pointers(dev_bufs))
+    hin = rank_pointer_array(host_in)
+    hout = rank_pointer_array(host_out)
+    dev = rank_pointer_array(dev_bufs)
     _check(_lib.gar_allreduce_host(plan.handle, hin, hout, dev, mode_c, _stream_handle(stream)),
            "gar_allreduce_host")
 
@@ -354,7 +372,7 @@ def gar_allreduce_batched(plans: Sequence[Plan], desc, count: int, stream=None) 
 
 
 def gar_allreduce_noalloc(plan: Plan, rank_buffers, stream=None) -> None:
-    ptrs = _ptr_array(rank_pointers(rank_buffers))
+    ptrs = rank_pointer_array(rank_buffers)
     _check(_lib.gar_allreduce_noalloc(plan.handle, ptrs, _stream_handle(stream)),
            "gar_allreduce_noalloc")
 
