@@ -277,9 +277,13 @@ def rank_pointer_array(rank_buffers) -> ctypes.Array:
         t = rank_buffers
         if t.stride(1) != 1:
             raise ValueError("rows must be contiguous")
-        a = (np.arange(t.shape[0], dtype=np.uint64) * np.uint64(t.stride(0) * t.element_size())
-             + np.uint64(t.data_ptr()))
+        P, base, step = t.shape[0], t.data_ptr(), t.stride(0) * t.element_size()
+        if P < 24:      # below about 24 ranks plain Python is faster than numpy
+            return (ctypes.c_void_p * P)(*[base + x * step for x in range(P)])
+        a = np.arange(P, dtype=np.uint64) * np.uint64(step) + np.uint64(base)
     elif len(rank_buffers) and isinstance(rank_buffers[0], int):
+        if len(rank_buffers) < 24:
+            return (ctypes.c_void_p * len(rank_buffers))(*rank_buffers)
         a = np.array(rank_buffers, dtype=np.uint64)
     else:
         a = np.array([int(b) if isinstance(b, int) else b.data_ptr() for b in rank_buffers],
