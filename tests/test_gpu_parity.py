@@ -94,6 +94,20 @@ def test_small_every_step_count(P, mode):
             _assert_same(got, want, dtype, f"P={P} n={n} {dtype} S={S} {mode}")
 
 
+@pytest.mark.parametrize("mode", ["fused", "step", "persistent"])
+def test_int32_wraparound(mode):
+    """int32 sums over the full value range overflow: every mode wraps modulo 2^32 like
+    the oracle (two's complement), at ragged small and chunked mid sizes, every S."""
+    for (P, n) in [(7, 1001), (24, 24 * 5003 + 11)]:
+        rng = np.random.default_rng(P)
+        t = torch.from_numpy(rng.integers(-2 ** 31, 2 ** 31, (P, n), dtype=np.int64).astype(np.int32))
+        host = _to_host_list(t, "i32")
+        for S in _Ss(P):
+            plan = gar.gar_plan_create(P, n, "i32", "sum", S)
+            _assert_same(_run(plan, t, mode), G.allreduce(host, S, "sum", "i32"), "i32",
+                         f"wrap P={P} n={n} S={S} {mode}")
+
+
 @pytest.mark.parametrize("P", [3, 7, 12])
 def test_mid_size_chunked_step_kernel(P):
     """Blocks of ~5000 elements with ragged starts: the chunked step-faithful launch
