@@ -135,6 +135,9 @@ __device__ __forceinline__ void *buf_ptr(const StepArgs<MAXP> &a, uint8_t buf, i
   return static_cast<char *>(a.ws[buf - BUF_QP0]) + (uint64_t)rank * a.n_pad * sizeof(A);
 }
 
+// v mod P for v in (-P, 2P).
+__device__ __forceinline__ int wrap_rank(int v, int P) { return v < 0 ? v + P : (v >= P ? v - P : v); }
+
 // This warp's slot of a step's byte counter.
 __device__ __forceinline__ int byte_slot() {
   return (int)((blockIdx.x * (kThreads / 32) + (threadIdx.x >> 5)) % STEP_BYTE_SLOTS);
@@ -155,13 +158,25 @@ struct LaunchView {
 template <typename T, int OP, int MAXP, bool kCopyPaths = true>
 __device__ __forceinline__ void chunk_work(const StepArgs<MAXP> &a, const LaunchView &lv, uint64_t item) {
   using A = typename AccOf<T>::type;
-  const int chunk = (int)(item % (uint64_t)lv.nchunks);
-  item /= (uint64_t)lv.nchunks;
-  const int x = (int)(item % (uint64_t)a.P);
-  const int oi = (int)(item / (uint64_t)a.P);
+  // 32-bit index arithmetic whenever the item fits (always for a launch's own grid):
+  // 64-bit division is a long software sequence and ran once per CTA.
+  int chunk, x, oi;
+  if (item <= 0xffffffffull) {
+    uint32_t it = (uint32_t)item;
+    chunk = (int)(it % (uint32_t)lv.nchunks);
+    it /= (uint32_t)lv.nchunks;
+    x = (int)(it % (uint32_t)a.P);
+    oi = (int)(it / (uint32_t)a.P);
+  } else {
+    chunk = (int)(item % (uint64_t)lv.nchunks);
+    item /= (uint64_t)lv.nchunks;
+    x = (int)(item % (uint64_t)a.P);
+    oi = (int)(item / (uint64_t)a.P);
+  }
   if (oi >= lv.nops) return;
   const StepOp op = lv.ops[oi];
-  const int b = a.xor_group ? (x ^ (int)op.dst_place) : ((x - (int)op.dst_place) % a.P + a.P) % a.P;
+  // placements and ranks are in [0, P), partner offsets in (-P, P)
+  const int b = a.xor_group ? (x ^ (int)op.dst_place) : wrap_rank(x - (int)op.dst_place, a.P);
   const uint64_t bstart = (uint64_t)b * a.q + ((uint64_t)b < a.rem ? (uint64_t)b : a.rem);
   const uint64_t blen = a.q + ((uint64_t)b < a.rem ? 1 : 0);
   const uint64_t c0 = (uint64_t)chunk * lv.chunk;
@@ -170,7 +185,7 @@ __device__ __forceinline__ void chunk_work(const StepArgs<MAXP> &a, const Launch
   const uint64_t hi = bstart + (blen < c0 + lv.chunk ? blen : c0 + lv.chunk);
 
   const bool has_recv = op.recv_place >= 0;
-  const int partner = a.xor_group ? (x ^ lv.partner) : ((x + lv.partner) % a.P + a.P) % a.P;
+  const int partner = a.xor_group ? (x ^ lv.partner) : wrap_rank(x + lv.partner, a.P);
   const void *recv = has_recv ? buf_ptr<A>(a, op.recv_buf, partner) : nullptr;
   void *out0 = buf_ptr<A>(a, op.out0_buf, x);
   const void *own0 = buf_ptr<A>(a, op.out0_own, x);
@@ -365,16 +380,30 @@ __device__ __forceinline__ void flat_work(const StepArgs<MAXP> &a, const LaunchV
   const uint64_t total = (uint64_t)lv.nops * a.n;
   const uint64_t big = a.rem * (a.q + 1);
   unsigned long long moved_bytes = 0;
+  // 32-bit index arithmetic when every index fits (the element-major launch serves
+  // short blocks, so practically always): 64-bit division is a long software sequence.
+  const bool narrow_idx = total + g_stride <= 0xffffffffull;
   for (uint64_t g = g_first; g < total; g += g_stride) {
-    const int oi = (int)(g / a.n);
-    const uint64_t e = g - (uint64_t)oi * a.n;
+    int oi, b;
+    uint64_t e;
+    if (narrow_idx) {
+      const uint32_t g32 = (uint32_t)g, n32 = (uint32_t)a.n;
+      oi = (int)(g32 / n32);
+      const uint32_t e32 = g32 - (uint32_t)oi * n32;
+      e = e32;
+      b = e32 < (uint32_t)big ? (int)(e32 / (uint32_t)(a.q + 1))
+                              : (int)((uint32_t)a.rem + (e32 - (uint32_t)big) / (uint32_t)a.q);
+    } else {
+      oi = (int)(g / a.n);
+      e = g - (uint64_t)oi * a.n;
+      b = e < big ? (int)(e / (a.q + 1)) : (int)(a.rem + (e - big) / a.q);
+    }
     const StepOp op = lv.ops[oi];
-    const int b = e < big ? (int)(e / (a.q + 1)) : (int)(a.rem + (e - big) / a.q);
-    const int x = a.xor_group ? (b ^ (int)op.dst_place) : (b + (int)op.dst_place) % a.P;
+    const int x = a.xor_group ? (b ^ (int)op.dst_place) : wrap_rank(b + (int)op.dst_place, a.P);
     A r = A(0);
     const bool has_recv = op.recv_place >= 0;
     if (has_recv) {
-      const int partner = a.xor_group ? (x ^ lv.partner) : ((x + lv.partner) % a.P + a.P) % a.P;
+      const int partner = a.xor_group ? (x ^ lv.partner) : wrap_rank(x + lv.partner, a.P);
       r = load1<T, A>(op.recv_buf, buf_ptr<A>(a, op.recv_buf, partner), e);
       moved_bytes += (op.recv_buf == BUF_RANK) ? sizeof(T) : sizeof(A);
     }
