@@ -34,6 +34,8 @@ def test_library_exports_every_declared_function():
     lib = ctypes.CDLL(gar.lib_path())
     for name in declared:
         assert hasattr(lib, name), name
+        # the binding has a wrapper of the same name for every entry point
+        assert callable(getattr(gar, name, None)), name
     # the binding's copies of the header's limits
     for name in ("GAR_MAX_P", "GAR_FUSED_MAX_OPS"):
         m = re.search(r"#define\s+" + name + r"\s+(\d+)", hdr)
