@@ -6,9 +6,12 @@
 // block index; eq. comm_op_0).  "Sending" is a coalesced 16-byte vector read of the
 // partner rank's block; the read value is combined in registers with the own block
 // (eq. distr_vectors_combination) and stored.  Every CTA owns one chunk of one block
-// of one (op, rank) pair.  Each warp counts the elements it read from partners and adds
-// the bytes to one of the step's counter slots, so the bytes a step actually moved are
-// recorded.
+// of one (op, rank) pair (short blocks: one thread per (op, element) instead).  Combine
+// ops batch 2 vectors per thread; same-type copies move raw 16-byte units, 6 per
+// thread; a bf16 plan's first step keeps its 16-byte bf16 loads packed until the
+// combine.  Each warp counts the elements it read from partners and adds the bytes to
+// one of the step's counter slots, so the bytes a step actually moved are recorded.
+// The launches of one Allreduce are chained by programmatic dependent launch.
 #include <cuda_bf16.h>
 #include <cuda_runtime.h>
 
