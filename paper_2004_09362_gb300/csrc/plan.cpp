@@ -24,6 +24,9 @@
 // ranks becomes XOR: placement p puts block i on rank i ^ p, the step operator is
 // t_{N_i/2} (x -> x ^ N_i/2), copy s has index k at placement s ^ k, and the unions of
 // the copies' placement sets are enumerated instead of taken as ranges.
+// Beyond 2L steps (cyclic group): fold schedules generalize the bandwidth-optimal step
+// from folding floor(N_i/2) vectors to folding f_i of them by t^{-f_i} (build_folds),
+// and the Ring moves one vector per step by the generator t (build_ring).
 #include <algorithm>
 #include <map>
 #include <stdexcept>
