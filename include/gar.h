@@ -286,14 +286,20 @@ GAR_API const char *gar_last_error(void);
  *   L < S < 2L:          eq. intemediate_cost  (2L-r) alpha + (2(P-1) + (2^r-1)(L-1)) u beta
  *                                              + ((P-1) + (2^r-1)(2L-2)) u gamma
  *   S = L (r = L):       eq. lo_cost           L alpha + P L u beta + P (2L-2) u gamma
- * with L = ceil(log2 P), r = 2L - S, m_bytes = bytes per rank.  Host-only.  Returns
- * GAR_EINVAL for P < 1 or S outside [L, 2L]. */
+ * with L = ceil(log2 P), r = 2L - S, m_bytes = bytes per rank; beyond 2L:
+ *   GAR_STEPS_RING:      eq. naive_cost        2(P-1) alpha + 2(P-1) u beta + (P-1) u gamma
+ *   fold schedule, even S in (2L, 2(P-1)]:     S alpha + 2(P-1) u beta + (P-1) u gamma
+ *     (the bandwidth-optimal traffic and combines in S steps; it equals eq. bo_cost at
+ *     S = 2L and eq. naive_cost at S = 2(P-1)).
+ * steps may be GAR_STEPS_BO / GAR_STEPS_LO.  Host-only.  Returns GAR_EINVAL for P < 1
+ * or a step count the plans do not take. */
 GAR_API int gar_cost_model(int P, int steps, double m_bytes, double alpha, double beta,
                            double gamma, double *tau);
 
 /* The step count minimising gar_cost_model over the integers S in [L, 2L] (eq.
  * opt_number_of_steps gives the continuous optimum in log P; the library takes the
- * integer argmin, smallest S on ties).  Host-only. */
+ * integer argmin, smallest S on ties).  Longer schedules are never cheaper in this model
+ * (same traffic as S = 2L, more alpha terms).  Host-only. */
 GAR_API int gar_optimal_steps(int P, double m_bytes, double alpha, double beta, double gamma,
                               int *steps);
 

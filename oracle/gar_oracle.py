@@ -702,15 +702,21 @@ def kahan_sum_f64(inputs) -> tuple[np.ndarray, np.ndarray]:
 # Cost model (Sec. "Communication model"; eqs. bo_cost, intemediate_cost, lo_cost)
 # ---------------------------------------------------------------------------
 
-def cost_model_time(P: int, m_bytes: float, steps: int, alpha: float, beta: float,
+def cost_model_time(P: int, m_bytes: float, steps, alpha: float, beta: float,
                     gamma: float) -> float:
     """tau for the version with S = steps (eq. bo_cost for r = 0, eq. intemediate_cost
-    for 0 < r < L, eq. lo_cost for r = L), with u = m/P."""
+    for 0 < r < L, eq. lo_cost for r = L), with u = m/P.  steps="ring": eq. naive_cost.
+    An even S in (2L, 2(P-1)], a fold schedule (reading C19), sends what the
+    bandwidth-optimal version sends and combines as often, in S steps."""
     L = ceil_log2(P)
+    u = m_bytes / P
+    if steps == "ring":
+        return 2 * (P - 1) * alpha + 2 * (P - 1) * u * beta + (P - 1) * u * gamma
+    if 2 * L < steps <= 2 * (P - 1) and steps % 2 == 0:
+        return steps * alpha + 2 * (P - 1) * u * beta + (P - 1) * u * gamma
     r = 2 * L - steps
     if not 0 <= r <= L:
         raise ValueError("steps out of range")
-    u = m_bytes / P
     if r == L:
         return L * alpha + P * L * u * beta + P * (2 * L - 2) * u * gamma
     return ((2 * L - r) * alpha

@@ -723,12 +723,24 @@ int gar_cost_model(int P, int steps, double m_bytes, double alpha, double beta, 
     return GAR_EINVAL;
   }
   const int L = ceil_log2(P);
+  const double u = m_bytes / P;
+  if (steps == GAR_STEPS_BO) steps = 2 * L;
+  if (steps == GAR_STEPS_LO) steps = L;
+  if (steps == GAR_STEPS_RING) {  // eq. naive_cost
+    *tau = 2.0 * (P - 1) * alpha + 2.0 * (P - 1) * u * beta + (P - 1) * u * gamma;
+    return GAR_OK;
+  }
+  if (steps > 2 * L && steps <= 2 * (P - 1) && steps % 2 == 0) {
+    // fold schedule: the bandwidth-optimal traffic and combines in S steps (equals
+    // eq. bo_cost at S = 2L and eq. naive_cost at S = 2(P-1))
+    *tau = steps * alpha + 2.0 * (P - 1) * u * beta + (P - 1) * u * gamma;
+    return GAR_OK;
+  }
   const int r = 2 * L - steps;
   if (r < 0 || r > L) {
-    set_error("steps outside [L, 2L]");
+    set_error("steps outside [L, 2L], an even count up to 2(P-1), or GAR_STEPS_*");
     return GAR_EINVAL;
   }
-  const double u = m_bytes / P;
   if (r == L) {  // latency-optimal, eq. lo_cost
     *tau = L * alpha + (double)P * L * u * beta + (double)P * (2.0 * L - 2.0) * u * gamma;
   } else {       // eq. intemediate_cost (r = 0 gives eq. bo_cost)

@@ -770,3 +770,26 @@ def test_oracle_order_free_results_equal_column_reduce(P):
             for o in G.allreduce(xs, S, op, dt, group=group):
                 np.testing.assert_array_equal(o, want, err_msg=f"P={P} S={S} {group} {dt} {op}")
 
+
+@pytest.mark.parametrize("P", [3, 5, 8, 24, 33, 127])
+def test_cost_model_beyond_2L_joins_the_paper_equations(P):
+    """Fold schedules cost S alpha plus the bandwidth-optimal traffic and combines: the
+    first fold (S = 2L + 2) is eq. bo_cost plus exactly two alpha terms, the last
+    (S = 2(P - 1)) is eq. naive_cost, the Ring's, and the traffic terms of every fold
+    are those the oracle's fold simulation sends (2(P - 1) blocks per rank)."""
+    L = G.ceil_log2(P)
+    m = 9.0 * 1024 * P
+    for (a, b, c) in [(1e-5, 1e-9, 1e-10), (2.5e-6, 0.0, 3e-13), (0.0, 1e-9, 0.0)]:
+        ring = G.cost_model_time(P, m, "ring", a, b, c)
+        if 2 * (P - 1) > 2 * L:
+            first = G.cost_model_time(P, m, 2 * L + 2, a, b, c)
+            assert first == pytest.approx(G.cost_model_time(P, m, 2 * L, a, b, c) + 2 * a, rel=1e-12, abs=1e-300)
+            assert G.cost_model_time(P, m, 2 * (P - 1), a, b, c) == pytest.approx(ring, rel=1e-12, abs=1e-300)
+    n = 7 * P
+    for S in range(2 * L + 2, 2 * (P - 1) + 1, 2):
+        run = G.simulate(P, n, S)
+        # all ranks together send 2(P - 1) n 4 bytes; the beta-only model per rank,
+        # 2(P - 1) u with u = m / P and m = 4 n, is that total over P
+        assert sum(run.step_bytes()) == 2 * (P - 1) * n * 4
+        assert G.cost_model_time(P, n * 4.0, S, 0.0, 1.0, 0.0) == pytest.approx(sum(run.step_bytes()) / P)
+

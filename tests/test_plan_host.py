@@ -417,8 +417,20 @@ def test_cost_model_matches_oracle():
                     assert gar.gar_cost_model(P, S, m, a, b, c) == pytest.approx(
                         G.cost_model_time(P, m, S, a, b, c), rel=1e-12, abs=1e-300)
                 assert gar.gar_optimal_steps(P, m, a, b, c) == G.optimal_steps(P, m, a, b, c)
+                # beyond 2L: fold schedules and the Ring; the BO / LO sentinels
+                for S in range(2 * L + 2, 2 * (P - 1) + 1, 2):
+                    assert gar.gar_cost_model(P, S, m, a, b, c) == pytest.approx(
+                        G.cost_model_time(P, m, S, a, b, c), rel=1e-12, abs=1e-300)
+                assert gar.gar_cost_model(P, gar.GAR_STEPS_RING, m, a, b, c) == pytest.approx(
+                    G.cost_model_time(P, m, "ring", a, b, c), rel=1e-12, abs=1e-300)
+                assert gar.gar_cost_model(P, gar.GAR_STEPS_BO, m, a, b, c) == \
+                    gar.gar_cost_model(P, 2 * L, m, a, b, c)
+                assert gar.gar_cost_model(P, gar.GAR_STEPS_LO, m, a, b, c) == \
+                    gar.gar_cost_model(P, L, m, a, b, c)
     with pytest.raises(gar.GarError):
         gar.gar_cost_model(8, 2, 1.0, 1.0, 1.0, 1.0)
+    with pytest.raises(gar.GarError):
+        gar.gar_cost_model(24, 13, 1.0, 1.0, 1.0, 1.0)     # odd, beyond 2L
 
 
 @pytest.mark.parametrize("P", [1, 2, 3, 4, 5, 7, 8, 13, 24, 33])
