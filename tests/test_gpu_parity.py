@@ -609,6 +609,31 @@ def test_host_buffers(P, n, dtype, S, mode, layout):
     assert bool((host_in[:, off:] == t).all())        # inputs untouched
 
 
+@pytest.mark.parametrize("mode", ["fused", "step", "persistent"])
+def test_host_buffers_other_schedules(mode):
+    """gar_allreduce_host with every schedule family: a fold schedule, the Ring and the
+    XOR group (pinned, aligned rows), and persistent mode on the copy path."""
+    for (P, n, dtype, steps, group, want_S) in [(24, 24 * 3001 + 5, "f32", 22, "cyclic", 22),
+                                                (8, 8 * 2001 + 3, "bf16", gar.GAR_STEPS_RING, "cyclic", "ring"),
+                                                (16, 16 * 4001, "f32", 6, "xor", 6)]:
+        t = _np_inputs(P, n, dtype, seed=17 + P)
+        per16 = 16 // t.element_size()
+        n_pad = (n + per16 - 1) // per16 * per16
+        host_in = torch.zeros((P, n_pad), dtype=t.dtype)
+        host_in[:, :n] = t
+        host_out = torch.zeros_like(host_in)
+        host_in, host_out = host_in.pin_memory(), host_out.pin_memory()
+        dev_store, _ = _padded_device(t)
+        plan = gar.gar_plan_create_group(P, n, dtype, "sum", steps, group)
+        rows_in = [host_in[x, :n] for x in range(P)]
+        rows_out = [host_out[x, :n] for x in range(P)]
+        gar.gar_allreduce_host(plan, rows_in, rows_out, dev_store, mode)
+        torch.cuda.synchronize()
+        want = G.allreduce(_to_host_list(t, dtype), want_S, "sum", dtype, group=group)
+        _assert_same(host_out[:, :n], want, dtype, f"host P={P} {group} S={want_S} {mode}")
+        assert bool((host_in[:, :n] == t).all())
+
+
 def test_missing_workspace_is_an_error():
     P, n = 7, 100
     plan = gar.gar_plan_create(P, n, "f32", "sum", 3)
