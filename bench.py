@@ -733,9 +733,9 @@ def run_reference(args):
     if rank != 0:
         return
     P, S = 24, 10
-    # size one step to ~(budget / steps) seconds
-    budget = 150.0
-    per_step = max(1.0, min(20.0, budget / max(1, args.steps + args.warmup)))
+    # size one step to ~(budget / steps) seconds (default budget 150 s)
+    budget = 15.0 * args.cpu_seconds
+    per_step = max(0.05, min(20.0, budget / max(1, args.steps + args.warmup)))
     n = 24 * 4096
     dt = _oracle_time(P, n, S)
     while dt < per_step / 2 and n * 2 <= 16777216:
