@@ -149,10 +149,6 @@ int check_buffers(const gar_plan *pl, void *const *bufs) {
 }
 
 int grid_for(const JitKernel *k, uint64_t work_items) {
-  int dev = 0, sms = 0;
-  cudaGetDevice(&dev);
-  cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
-  if (sms <= 0) sms = 1;
   // One work item per thread: with many more CTAs than fit at once the block scheduler
   // keeps every SM full and each thread's loads are in flight together (a persistent
   // grid-stride loop serialises a thread's iterations and ran 6% slower on GB300).
@@ -161,8 +157,13 @@ int grid_for(const JitKernel *k, uint64_t work_items) {
   const uint64_t need = (work_items + k->threads - 1) / k->threads;
   uint64_t cap = 0x7fffffffull;
   const char *wv = std::getenv("GAR_TUNE_GRID_WAVES");
-  if (wv && std::atoi(wv) > 0)
+  if (wv && std::atoi(wv) > 0) {
+    int dev = 0, sms = 0;
+    cudaGetDevice(&dev);
+    cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
+    if (sms <= 0) sms = 1;
     cap = (uint64_t)sms * (uint64_t)std::max(1, k->blocks_per_sm) * (uint64_t)std::atoi(wv);
+  }
   return (int)std::max<uint64_t>(1, std::min<uint64_t>(need, cap));
 }
 
