@@ -468,3 +468,18 @@ def test_ring_plan_matches_oracle(P):
                 np.testing.assert_array_equal(got[x].view(np.uint32), want[x].view(np.uint32))
     with pytest.raises(gar.GarError):
         gar.gar_plan_create_group(8, 10, "f32", "sum", gar.GAR_STEPS_RING, "xor")
+
+
+@pytest.mark.parametrize("P,n", [(24, 16777216), (5, 1024), (7, 1001), (127, 4194304), (2, 33)])
+def test_bench_dram_model_closed_form(P, n):
+    """bench.py's step-faithful DRAM model (bytes the kernels read and write, counted
+    from the op tables) against a closed form: bandwidth-optimal fp32 combines every
+    element position P - 1 times (partner read + own read + write, 12 B) and copies it
+    P - 1 times (read + write, 8 B): (P - 1) * n * 20 bytes.  For P = 24 x 16 Mi that is
+    the 7,717,519,360 B the bench reports."""
+    import importlib.util
+    spec = importlib.util.spec_from_file_location("bench_mod", os.path.join(ROOT, "bench.py"))
+    bench = importlib.util.module_from_spec(spec)
+    spec.loader.exec_module(bench)
+    plan = gar.gar_plan_create(P, n, "f32", "sum", gar.GAR_STEPS_BO)
+    assert bench._step_dram_bytes(gar, plan, P, n, "f32") == (P - 1) * n * 20
