@@ -8,7 +8,7 @@ two share no code: the only common dependency is the seeded input generator modu
 
 See ``oracle/gar_oracle.py`` for what is computed and which passage of the paper each
 function follows.  Parity status: every function here is pinned by ``-m "not gpu"``
-tests (``tests/test_oracle_pins.py``) except where a docstring says "parity unpinned".
+tests (``tests/test_oracle_pins.py``); each docstring names its pins ("Pinned by:").
 """
 
 from .gar_oracle import *  # noqa: F401,F403

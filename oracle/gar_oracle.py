@@ -91,7 +91,10 @@ _ACC_ITEMSIZE = {"f32": 4, "bf16": 4, "i32": 4}
 
 def ceil_log2(P: int) -> int:
     """L = ceil(log2 P): the number of reduction steps (Sec. "Bandwidth-optimal
-    algorithm": the reduction phase takes ceil(log P) steps)."""
+    algorithm": the reduction phase takes ceil(log P) steps).
+
+    Pinned by: test_step_counts.
+    """
     if P < 1:
         raise ValueError("P must be >= 1")
     L = 0
@@ -102,7 +105,10 @@ def ceil_log2(P: int) -> int:
 
 def vector_counts(P: int) -> list[int]:
     """[N_0, ..., N_L] with N_0 = P and N_{i+1} = ceil(N_i / 2) (eq.
-    bo_starting_set_size)."""
+    bo_starting_set_size).
+
+    Pinned by: test_step_counts, test_planted_floor_halving_is_caught.
+    """
     Ns = [P]
     while Ns[-1] > 1:
         Ns.append((Ns[-1] + 1) // 2)
@@ -112,7 +118,11 @@ def vector_counts(P: int) -> list[int]:
 def block_bounds(n: int, P: int) -> list[tuple[int, int]]:
     """Block i of every vector (eq. initial_data).  The paper assumes equal blocks
     u = m/P (Sec. "Communication model"); for P not dividing n the first n mod P blocks
-    get one extra element (reading C3)."""
+    get one extra element (reading C3).
+
+    Pinned by: test_block_bounds_reading_c3 (hand-written sizes),
+    test_planted_partition_mistake_is_caught.
+    """
     q, rem = divmod(n, P)
     out, start = [], 0
     for i in range(P):
@@ -129,7 +139,10 @@ def schedule_shape(P: int, steps: int) -> dict:
     number K of q_Sigma copies the reduction phase must end with (reading C7:
     K = N_{L-r}).  Even S in (2L, 2(P-1)] selects the fold schedule (fold_sequence;
     K = 1), the step counts toward the Ring that Sec. "Conclusion" leaves to future work
-    (reading C19)."""
+    (reading C19).
+
+    Pinned by: test_step_counts, test_fold_schedule.
+    """
     L = ceil_log2(P)
     if L <= steps <= 2 * L:
         r = 2 * L - steps
@@ -147,7 +160,10 @@ def fold_sequence(P: int, F: int) -> list[int]:
     and combines them there; f = floor(N/2) is the bandwidth-optimal step (eqs.
     bo_tx_dist, bo_dir_perms), f = 1 moves one vector by the generator.  F = L gives the
     bandwidth-optimal halving; F > L spreads the P-1 folds as evenly as the constraints
-    allow (1 <= f <= floor(N/2), and the remaining steps must still reach N = 1)."""
+    allow (1 <= f <= floor(N/2), and the remaining steps must still reach N = 1).
+
+    Pinned by: test_fold_schedule, test_fold_schedule_ends.
+    """
     L = ceil_log2(P)
     if not (L <= F <= max(P - 1, L)):
         raise ValueError("F out of range")
@@ -174,7 +190,11 @@ def fold_sequence(P: int, F: int) -> list[int]:
 class ExprTable:
     """Interned contents.  A leaf k is the initial vector t_k q_k (block i from process
     i + k, eq. initial_distr_vector); a pair (a, b) is the combination "own (+)
-    received" of two same-placement vectors (eq. distr_vectors_combination)."""
+    received" of two same-placement vectors (eq. distr_vectors_combination).
+
+    Pinned by: test_golden_tree (hand-derived trees),
+    test_every_output_covers_every_rank_once.
+    """
 
     def __init__(self):
         self.nodes: list = []          # id -> ("leaf", k) | ("pair", a, b)
@@ -217,14 +237,20 @@ class ExprTable:
 
 
 def tree_string(t) -> str:
-    """'(a+b)' notation for a nested-tuple tree; leaves are integers."""
+    """'(a+b)' notation for a nested-tuple tree; leaves are integers.
+
+    Pinned by: test_tree_notation_round_trip.
+    """
     if isinstance(t, int):
         return str(t)
     return "(" + tree_string(t[0]) + "+" + tree_string(t[1]) + ")"
 
 
 def parse_tree(s: str):
-    """Inverse of tree_string (used for the hand-derived fixtures in tests/golden)."""
+    """Inverse of tree_string (used for the hand-derived fixtures in tests/golden).
+
+    Pinned by: test_tree_notation_round_trip.
+    """
     s = s.replace(" ", "")
     pos = 0
 
@@ -251,7 +277,10 @@ def parse_tree(s: str):
 
 def eval_tree(t, leaf_value, op: str):
     """Evaluate a nested-tuple tree with leaf_value(k) at the leaves, combining with op
-    in whatever numpy type the leaves carry."""
+    in whatever numpy type the leaves carry.
+
+    Pinned by: test_golden_tree_values.
+    """
     if isinstance(t, int):
         return leaf_value(t)
     return _combine(op, eval_tree(t[0], leaf_value, op), eval_tree(t[1], leaf_value, op))
@@ -260,7 +289,11 @@ def eval_tree(t, leaf_value, op: str):
 def group_ops(P: int, group: str):
     """(op, inverse) of the permutation group T_P acting on {0..P-1}: t_a(t_b(x)) =
     op(op(x, b), a).  "cyclic": t_k(x) = x + k mod P (Table 1a); "xor": t_k(x) = x XOR k,
-    the self-inverse group generated by the h_i of Table 1b (P a power of two)."""
+    the self-inverse group generated by the h_i of Table 1b (P a power of two).
+
+    Pinned by: test_xor_group_bo_is_recursive_halving,
+    test_xor_group_lo_is_recursive_doubling.
+    """
     if group == "cyclic":
         return (lambda a, b: (a + b) % P), (lambda a: (-a) % P)
     if group == "xor":
@@ -273,21 +306,30 @@ def group_ops(P: int, group: str):
 def _reduce_partner(x: int, d: int, P: int, group: str = "cyclic") -> int:
     """Where process x sends during a reduction step: the step operator
     t_d^{-1} (t^{-d} in the cyclic group, eqs. comm_op_0, bo_dir_perms) moves every
-    block from x to t_d^{-1}(x)."""
+    block from x to t_d^{-1}(x).
+
+    Pinned by: test_tx_sets_and_partners, test_planted_wrong_partner_is_caught.
+    """
     op, inv = group_ops(P, group)
     return op(x, inv(d))
 
 
 def _distribute_partner(x: int, d: int, P: int, group: str = "cyclic") -> int:
     """Where process x sends during a distribution step: the reversed operator t_d
-    (t^{+d} in the cyclic group; end of Sec. "Bandwidth-optimal algorithm")."""
+    (t^{+d} in the cyclic group; end of Sec. "Bandwidth-optimal algorithm").
+
+    Pinned by: test_int32_bruteforce, test_ring_equals_textbook_ring.
+    """
     op, _inv = group_ops(P, group)
     return op(x, d)
 
 
 def _combine(op: str, a, b):
     """The reduction operator (+) of the Allreduce (Sec. "Combination of distributed
-    data vectors"); elementwise, in the operands' own numpy type."""
+    data vectors"); elementwise, in the operands' own numpy type.
+
+    Pinned by: test_int32_bruteforce, test_planted_sign_error_is_caught.
+    """
     if op == "sum":
         return a + b
     if op == "max":
@@ -304,7 +346,10 @@ def _combine(op: str, a, b):
 def round_to_bf16(x: np.ndarray) -> np.ndarray:
     """Round float32 values to the nearest bfloat16 (ties to even), returned as float32.
     bfloat16 keeps the top 16 bits of the float32 encoding (sign, 8 exponent bits,
-    7 fraction bits); rounding looks at the 16 discarded bits.  Finite inputs only."""
+    7 fraction bits); rounding looks at the 16 discarded bits.  Finite inputs only.
+
+    Pinned by: test_bf16_rounding_matches_library (torch's conversion).
+    """
     x = np.ascontiguousarray(x, dtype=np.float32)
     bits = x.view(np.uint32).astype(np.uint64)
     upper = bits >> np.uint64(16)
@@ -327,7 +372,10 @@ def is_bf16_exact(x: np.ndarray) -> bool:
 
 @dataclass
 class Run:
-    """Everything one simulated Allreduce produced."""
+    """Everything one simulated Allreduce produced.
+
+    Pinned by: test_is_bf16_exact.
+    """
     P: int
     n: int
     steps: int
@@ -381,6 +429,8 @@ def simulate(P: int, n: int, steps: int, inputs=None, op: str = "sum",
     elements: optional sorted array of global element indices; the run then carries
       only those elements (every operation is elementwise, so they come out exactly as
       in a full run).  Message sizes are always those of the full vectors.
+
+    Pinned by: every test in tests/test_oracle_pins.py.
     """
     if op not in OPS:
         raise ValueError(op)
@@ -564,7 +614,10 @@ def simulate_ring(P: int, n: int, inputs=None, op: str = "sum", dtype: str = "f3
     placement i moves by t to placement i + 1 and is combined with the initial vector
     t^{i+1} q_{i+1} there (eq. ring_reduce: own t^{i+1} q_{i+1} (+) received).  After P-1
     steps placement P-1 holds q_Sigma; the distribution phase moves copies by t again,
-    P-1 more steps (2(P-1) in total, eq. naive_cost)."""
+    P-1 more steps (2(P-1) in total, eq. naive_cost).
+
+    Pinned by: test_ring_equals_textbook_ring, test_ring_steps_traffic_and_tree.
+    """
     if op not in OPS:
         raise ValueError(op)
     if dtype not in DTYPES:
@@ -652,7 +705,10 @@ def allreduce(inputs, steps: int, op: str = "sum", dtype: str = "f32", elements=
               group: str = "cyclic"):
     """MPI_Allreduce semantics (Sec. "Introduction"): every process ends with the
     op-reduction of all P input vectors.  Returns the list of P output arrays (over the
-    selected elements when ``elements`` is given)."""
+    selected elements when ``elements`` is given).
+
+    Pinned by: test_int32_bruteforce, test_float_max_min_exact, test_golden_tree_values.
+    """
     P = len(inputs)
     n = len(inputs[0]) if P else 0
     if steps == "ring":
@@ -669,7 +725,10 @@ def column_reduce_exact(inputs, op: str, dtype: str):
     """The Allreduce result from its definition, u_{i,Sigma} = u_{i,0} (+) ... (+)
     u_{i,P-1} (Sec. "Combination of distributed data vectors"), for the cases where it
     has a unique value: i32 sum in exact integers reduced mod 2^32 (two's complement),
-    and max/min of any type."""
+    and max/min of any type.
+
+    Pinned by: test_column_reduce_exact_brute_force (pure-Python loops).
+    """
     stack = np.stack([np.asarray(v) for v in inputs])
     if op == "sum":
         if dtype != "i32":
@@ -686,7 +745,11 @@ def column_reduce_exact(inputs, op: str, dtype: str):
 
 def kahan_sum_f64(inputs) -> tuple[np.ndarray, np.ndarray]:
     """Compensated (Kahan) sum of the P inputs in rank order, in float64, and the sum
-    of absolute values (the scale of the standard summation error bound)."""
+    of absolute values (the scale of the standard summation error bound).
+
+    Pinned by: test_kahan_sum_within_compensated_bound (math.fsum),
+    test_kahan_sum_recovers_lost_low_bits, test_planted_kahan_sign_flip_is_caught.
+    """
     stack = np.stack([np.asarray(v, dtype=np.float64) for v in inputs])
     s = np.zeros(stack.shape[1], dtype=np.float64)
     comp = np.zeros_like(s)
@@ -707,7 +770,12 @@ def cost_model_time(P: int, m_bytes: float, steps, alpha: float, beta: float,
     """tau for the version with S = steps (eq. bo_cost for r = 0, eq. intemediate_cost
     for 0 < r < L, eq. lo_cost for r = L), with u = m/P.  steps="ring": eq. naive_cost.
     An even S in (2L, 2(P-1)], a fold schedule (reading C19), sends what the
-    bandwidth-optimal version sends and combines as often, in S steps."""
+    bandwidth-optimal version sends and combines as often, in S steps.
+
+    Pinned by: test_cost_model_argmin_matches_paper_example,
+    test_cost_model_beyond_2L_joins_the_paper_equations,
+    test_bandwidth_optimal_traffic.
+    """
     L = ceil_log2(P)
     u = m_bytes / P
     if steps == "ring":
@@ -726,7 +794,10 @@ def cost_model_time(P: int, m_bytes: float, steps, alpha: float, beta: float,
 
 def optimal_steps(P: int, m_bytes: float, alpha: float, beta: float, gamma: float) -> int:
     """The step count minimising the cost model over integer S in [L, 2L] (eq.
-    opt_number_of_steps gives the continuous optimum; reading C15 takes the argmin)."""
+    opt_number_of_steps gives the continuous optimum; reading C15 takes the argmin).
+
+    Pinned by: test_cost_model_argmin_matches_paper_example.
+    """
     L = ceil_log2(P)
     if L == 0:
         return 0

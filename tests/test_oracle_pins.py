@@ -32,6 +32,15 @@ def _golden():
     return rows
 
 
+def _mpi_partition(n, P):
+    """Block boundaries written out here, independently of the oracle: MPI
+    reduce_scatter's split, where the first n mod P blocks are one element longer
+    (reading C3 of the paper's u = m/P, Sec. "Communication model", eq. initial_data)."""
+    q, rem = n // P, n % P
+    starts = [i * q + min(i, rem) for i in range(P + 1)]
+    return [(starts[i], starts[i + 1]) for i in range(P)]
+
+
 def _Ls(P):
     L = G.ceil_log2(P)
     return L, list(range(L, 2 * L + 1))
@@ -61,7 +70,7 @@ def test_golden_tree_values(row):
     xs = [(rng.standard_normal(n) * np.exp2(rng.integers(-20, 21, n))).astype(np.float32)
           for _ in range(P)]
     run = G.simulate(P, n, S, inputs=xs, op="sum", dtype="f32")
-    bounds = G.block_bounds(n, P)
+    bounds = _mpi_partition(n, P)
     for x in range(P):
         for b in range(P):
             if (x - b) % P != p:
@@ -329,6 +338,182 @@ def test_bo_all_ranks_identical_and_lo_rotated():
 
 
 # ---------------------------------------------------------------------------
+# Block partition (eq. initial_data with u = m/P, Sec. "Communication model";
+# reading C3 for P not dividing n)
+# ---------------------------------------------------------------------------
+
+# (n, P, block sizes in order), written out by hand from reading C3: the first n mod P
+# blocks get one element more than floor(n / P); n < P leaves the last blocks empty.
+BLOCK_SIZES = [
+    (1024, 5, [205, 205, 205, 205, 204]),
+    (16_777_216, 24, [699_051] * 16 + [699_050] * 8),
+    (4_194_304, 127, [33_027] * 2 + [33_026] * 125),
+    (262_144, 8, [32_768] * 8),
+    (3, 5, [1, 1, 1, 0, 0]),
+    (0, 4, [0, 0, 0, 0]),
+    (7, 1, [7]),
+    (106, 6, [18, 18, 18, 18, 17, 17]),
+    (106, 7, [16] * 1 + [15] * 6),
+]
+
+
+@pytest.mark.parametrize("n,P,sizes", BLOCK_SIZES, ids=lambda v: str(v) if not isinstance(v, list) else "")
+def test_block_bounds_reading_c3(n, P, sizes):
+    """Block i is [sum of sizes before i, + sizes[i]): contiguous, in block order, from 0
+    to n, with the sizes written out above."""
+    assert sum(sizes) == n and len(sizes) == P
+    bounds = G.block_bounds(n, P)
+    assert len(bounds) == P
+    start = 0
+    for (lo, hi), size in zip(bounds, sizes):
+        assert (lo, hi) == (start, start + size)
+        start += size
+    assert start == n
+
+
+def _block_pins_pass() -> bool:
+    try:
+        for n, P, sizes in BLOCK_SIZES:
+            test_block_bounds_reading_c3(n, P, sizes)
+    except AssertionError:
+        return False
+    return True
+
+
+def _remainder_last(n, P):
+    q, rem = divmod(n, P)
+    out, start = [], 0
+    for i in range(P):
+        size = q + (1 if i >= P - rem else 0)
+        out.append((start, start + size))
+        start += size
+    return out
+
+
+def _remainder_in_last_block(n, P):
+    q, rem = divmod(n, P)
+    out = [(i * q, (i + 1) * q) for i in range(P)]
+    out[-1] = (out[-1][0], n)
+    return out
+
+
+@pytest.mark.parametrize("bad", [_remainder_last, _remainder_in_last_block])
+def test_planted_partition_mistake_is_caught(monkeypatch, bad):
+    """Two plausible misreadings of reading C3 -- the longer blocks at the end, or the
+    whole remainder in block P-1 -- fail the hand-written sizes, and they also change
+    the simulation's results against checkers that partition on their own (the golden
+    tree values and the textbook Ring below).  (Recursive Halving cannot see it: its
+    tree is the same butterfly for every block.)"""
+    monkeypatch.setattr(G, "block_bounds", bad)
+    assert not _block_pins_pass()
+    row = next(r for r in _golden() if r[1] == 7)
+    with pytest.raises(AssertionError):
+        test_golden_tree_values(row)
+    with pytest.raises(AssertionError):
+        test_ring_equals_textbook_ring(5)
+
+
+def test_tree_notation_round_trip():
+    """The fixture notation of tests/golden: hand-written strings and their trees."""
+    cases = {"3": 3, "(0+1)": (0, 1), "((0+1)+(2+(3+4)))": ((0, 1), (2, (3, 4))),
+             "(12+(0+7))": (12, (0, 7))}
+    for text, tree in cases.items():
+        assert G.parse_tree(text) == tree
+        assert G.tree_string(tree) == text
+
+
+def test_is_bf16_exact():
+    assert G.is_bf16_exact(np.float32([0.0, 1.0, -2.5, 2.0 ** 127, 2.0 ** -120, -1.5 * 2.0 ** 60]))
+    for v in (1.0 + 2.0 ** -8, 1.0 + 2.0 ** -23, 0.1):
+        assert not G.is_bf16_exact(np.float32([1.0, v]))
+
+
+def test_column_reduce_exact_brute_force():
+    """The definition, checked against pure-Python loops over tiny inputs: int32 sums
+    wrap modulo 2^32 (two's complement), max and min pick the extreme value."""
+    rng = np.random.default_rng(21)
+    for P in (1, 2, 5, 9):
+        xs = [rng.integers(-2**31, 2**31, 13, dtype=np.int64).astype(np.int32) for _ in range(P)]
+        for op in ("sum", "max", "min"):
+            got = G.column_reduce_exact(xs, op, "i32")
+            for e in range(13):
+                col = [int(x[e]) for x in xs]
+                if op == "sum":
+                    t = sum(col) & 0xFFFFFFFF
+                    want = t - 2**32 if t >= 2**31 else t
+                else:
+                    want = max(col) if op == "max" else min(col)
+                assert int(got[e]) == want
+        fs = [rng.standard_normal(13).astype(np.float32) for _ in range(P)]
+        for op in ("max", "min"):
+            got = G.column_reduce_exact(fs, op, "f32")
+            for e in range(13):
+                col = [float(x[e]) for x in fs]
+                assert float(got[e]) == (max(col) if op == "max" else min(col))
+
+
+# ---------------------------------------------------------------------------
+# The compensated reference sum (the Kahan reference of the float tolerance)
+# ---------------------------------------------------------------------------
+
+def _kahan_cases():
+    rng = np.random.default_rng(11)
+    cases = []
+    for P in (2, 5, 24, 127):
+        x = rng.standard_normal((P, 500)) * np.exp2(rng.integers(-30, 31, (P, 500)))
+        cases.append(x)
+    # heavy cancellation: large terms of both signs around small ones
+    big = rng.standard_normal((40, 300)) * 1e12
+    cases.append(np.concatenate([big, rng.standard_normal((40, 300)), -big[::-1]]))
+    return cases
+
+
+def test_kahan_sum_within_compensated_bound():
+    """Compensated summation of P terms has |error| <= (2u + O(P u^2)) sum|x| with
+    u = 2^-53 (the standard bound for Kahan's method); the exact sum comes from
+    math.fsum, which rounds the exact sum once.  A plain float64 sum of these inputs
+    does not meet the bound, so a broken compensation fails it."""
+    import math
+    u = 2.0 ** -53
+    for x in _kahan_cases():
+        P = x.shape[0]
+        s, mag = G.kahan_sum_f64(list(x))
+        exact = np.array([math.fsum(x[:, j]) for j in range(x.shape[1])])
+        want_mag = np.array([math.fsum(np.abs(x[:, j])) for j in range(x.shape[1])])
+        np.testing.assert_allclose(mag, want_mag, rtol=P * u, atol=0)
+        assert np.all(np.abs(s - exact) <= (2 * u + 2 * P * u * u) * want_mag)
+
+
+def test_kahan_sum_recovers_lost_low_bits():
+    """1 + 1000 * 2^-60: every addend is below half an ulp of 1, so rank-order plain
+    summation returns exactly 1.0, while compensated summation returns the correctly
+    rounded 1 + 1000 * 2^-60 (= 1 + 4 * 2^-52)."""
+    import math
+    col = [1.0] + [2.0 ** -60] * 1000
+    s, _ = G.kahan_sum_f64([np.array([v]) for v in col])
+    assert s[0] == math.fsum(col) == 1.0 + 4 * 2.0 ** -52
+
+
+def test_planted_kahan_sign_flip_is_caught(monkeypatch):
+    """The compensation term with its sign flipped (c = y - (t - s)) fails both pins."""
+    def flipped(inputs):
+        stack = np.stack([np.asarray(v, dtype=np.float64) for v in inputs])
+        s = np.zeros(stack.shape[1])
+        comp = np.zeros_like(s)
+        for row in stack:
+            y = row - comp
+            t = s + y
+            comp = y - (t - s)
+            s = t
+        return s, np.abs(stack).sum(axis=0)
+    monkeypatch.setattr(G, "kahan_sum_f64", flipped)
+    with pytest.raises(AssertionError):
+        test_kahan_sum_within_compensated_bound()
+    with pytest.raises(AssertionError):
+        test_kahan_sum_recovers_lost_low_bits()
+
+
+# ---------------------------------------------------------------------------
 # Floating point: error bounds and bf16
 # ---------------------------------------------------------------------------
 
@@ -482,7 +667,7 @@ def _textbook_recursive_halving(xs):
     index agrees with its own rank in the exchanged bit).  Written from the textbook
     description, independently of the oracle's schedule simulation."""
     P, n = len(xs), len(xs[0])
-    bounds = G.block_bounds(n, P)
+    bounds = _mpi_partition(n, P)
     buf = [x.copy() for x in xs]
     resp = [list(range(P)) for _ in range(P)]
     m = P // 2
@@ -596,7 +781,7 @@ def _textbook_ring(xs):
     chunk to it, then P-1 allgather steps passing the finished chunks on.  Written
     independently of the oracle's schedule simulation."""
     P, n = len(xs), len(xs[0])
-    bounds = G.block_bounds(n, P)
+    bounds = _mpi_partition(n, P)
     buf = [x.copy() for x in xs]
     for i in range(P - 1):
         new = [b.copy() for b in buf]
