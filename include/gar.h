@@ -129,7 +129,16 @@ typedef struct {
   int32_t fused_local_bytes; /* local (spill) bytes per thread of the loaded fused kernel */
   int32_t group;             /* GAR_GROUP_CYCLIC or GAR_GROUP_XOR */
   int32_t ring;              /* 1 for the Ring schedule (GAR_STEPS_RING) */
+  int32_t fused_form;        /* fused kernel the plan uses: GAR_FORM_SINGLE or GAR_FORM_BREADTH */
 } gar_plan_info;
+
+/* Values of gar_plan_info.fused_form.  GAR_FORM_SINGLE: each thread evaluates the whole
+ * program result by result for 1..8 element positions.  GAR_FORM_BREADTH: each thread
+ * evaluates it step by step for one element position, with paired fp32 adds; taken by
+ * float sums with several result copies whose single-thread form would keep more than
+ * 160 values alive per element position (large latency-optimal and near-latency-optimal
+ * schedules, e.g. P = 127 at S = 7 and 8).  Both give the same bits. */
+enum { GAR_FORM_SINGLE = 0, GAR_FORM_BREADTH = 1 };
 
 /* Creates a schedule for P virtual ranks of n elements each.
  * P: 1..GAR_MAX_P.  n: elements per rank (0 is allowed: every call is a no-op).

@@ -6,6 +6,7 @@
 #include <cstdlib>
 #include <cstring>
 #include <new>
+#include <stdexcept>
 #include <string>
 #include <vector>
 
@@ -103,10 +104,30 @@ int check_fused_size(const gar_plan *pl) {
   return GAR_OK;
 }
 
+// The fused kernel a plan uses.  Float sums with several result copies whose
+// single-thread program keeps more than 160 values alive per element position (P = 127
+// at S = 7 and 8: 254 and 192) are register-bound in that form and take the
+// breadth-first form (0.59 instead of 0.68 ms, and 0.47 instead of 0.56 ms, at P = 127 x
+// 8 MiB bf16 on GB300); every other plan takes the single-thread form.  GAR_TUNE_FUSED_FORM
+// (0 or 1) forces one form, for parity tests and launch-shape sweeps.
+CodegenResult fused_codegen(const gar_plan &pl) {
+  const char *ff = std::getenv("GAR_TUNE_FUSED_FORM");
+  int form = (pl.K > 1 && pl.op == GAR_SUM && pl.dtype != GAR_I32 && fused_peak_live(pl) > 160) ? 1 : 0;
+  if (ff && *ff) form = std::atoi(ff) == 1 ? 1 : 0;
+  if (form == 1 && pl.K > 1) return generate_fused_bf_source(pl);
+  return generate_fused_source(pl);
+}
+
 int compile_fused(gar_plan *pl) {
   if (pl->fused) return GAR_OK;
   if (int rc = check_fused_size(pl)) return rc;
-  CodegenResult cg = generate_fused_source(*pl);
+  CodegenResult cg;
+  try {
+    cg = fused_codegen(*pl);
+  } catch (const std::exception &ex) {
+    set_error(std::string("fused code generation: ") + ex.what());
+    return GAR_EINVAL;
+  }
   JitKernel *k = nullptr;
   int rc = jit_compile(cg, &k);
   if (rc) return rc;
@@ -440,6 +461,7 @@ int gar_plan_get_info(const gar_plan *pl, gar_plan_info *info) {
   info->fused_combines = (int)pl->prog.a.size();
   info->group = pl->group;
   info->ring = pl->ring ? 1 : 0;
+  info->fused_form = pl->K > 1 ? fused_codegen(*pl).form : GAR_FORM_SINGLE;
   info->fused_width = pl->fused_width;
   if (pl->fused != nullptr && pl->fused->loaded) {
     info->fused_regs = pl->fused->regs;
@@ -520,7 +542,13 @@ int gar_plan_step_ops(const gar_plan *pl, int32_t *ops, int *nops, int32_t *laun
 int gar_plan_fused_source(const gar_plan *pl, char *buf, size_t *len) {
   if (int rc = check_plan(pl)) return rc;
   if (len == nullptr) return GAR_EINVAL;
-  const std::string src = generate_fused_source(*pl).source;
+  std::string src;
+  try {
+    src = fused_codegen(*pl).source;
+  } catch (const std::exception &ex) {
+    set_error(std::string("fused code generation: ") + ex.what());
+    return GAR_EINVAL;
+  }
   if (buf != nullptr && *len > 0) {
     const size_t m = std::min(*len - 1, src.size());
     std::memcpy(buf, src.data(), m);

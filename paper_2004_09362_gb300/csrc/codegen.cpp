@@ -11,6 +11,8 @@
 #include <cstdio>
 #include <cstdlib>
 #include <functional>
+#include <map>
+#include <stdexcept>
 #include <string>
 #include <vector>
 
@@ -328,9 +330,13 @@ CodegenResult generate_fused_source(const gar_plan &pl) {
   if (int w = tune_int("GAR_TUNE_FUSED_W", 0))
     if (w > 0 && (w & (w - 1)) == 0 && w * elem_size(pl.dtype) <= 16) W = w;
   const int minb = tune_int("GAR_TUNE_FUSED_MINB", 0);
-  const std::string bounds = minb > 0 ? fmt("__launch_bounds__(256, %d)", minb) : "__launch_bounds__(256)";
+  int nthr = tune_int("GAR_TUNE_FUSED_THREADS", 256);
+  if (nthr < 32 || nthr > 1024 || nthr % 32 != 0) nthr = 256;
+  const std::string bounds = minb > 0 ? fmt("__launch_bounds__(%d, %d)", nthr, minb)
+                                      : fmt("__launch_bounds__(%d)", nthr);
   CodegenResult cg;
   cg.width = W;
+  cg.threads = nthr;
   cg.kernel_name = fmt("gar_fused_P%d_S%d_K%d_", P, pl.S, pl.K) + dtype_tag(pl.dtype) + "_" +
                    op_tag(pl.op) + fmt("_W%d", W) + (pl.group == GAR_GROUP_XOR ? "_xor" : "");
   std::string s;
@@ -402,6 +408,244 @@ CodegenResult generate_fused_source(const gar_plan &pl) {
   cg.source = s;
   return cg;
 }
+
+// ---------------------------------------------------------------------------
+// Breadth-first fused kernel, for programs whose single-thread form is register-bound.
+//
+// With many result copies the schedule keeps a q' and a q* vector at most placements
+// (Sec. "Latency-optimal version"): at P = 127, S = 7 about 2P = 254 values per element
+// position are alive at once, the kernel above spills and runs one 256-thread CTA per
+// SM.  This form evaluates the same program step by step instead of result by result:
+//  * every contribution is loaded at the start, so a warp waits for memory once;
+//  * the combines of one step (which never depend on each other) follow in placement
+//    order, which leaves the compiler long independent runs to schedule;
+//  * in float sums, two combines whose placements, operands and results form adjacent
+//    pairs run as one paired fp32 add (__fadd2_rn: round to nearest even in each half);
+//  * bf16 contributions enter a sum through the mixed-precision add.rn.f32.bf16 (the
+//    bf16 value widens exactly, one rounding), so they are never unpacked separately;
+//  * small CTAs (32 or 64 threads), several per SM, so the CTAs of an SM drift apart and
+//    one's loads overlap another's combines.
+// Both adds round exactly as the scalar fp32 add does, so the bits are the schedule's.
+// ---------------------------------------------------------------------------
+
+namespace {
+
+const char *kBFHelpers = R"CUDA(
+static __device__ __forceinline__ gar_acc gar_wide(gar_io x) {
+#if GAR_DTYPE == 1
+  return __uint_as_float(((gar_u32)x) << 16);
+#else
+  return x;
+#endif
+}
+static __device__ __forceinline__ gar_io gar_ldio(const gar_io *p) {
+  gar_io v;
+#if GAR_DTYPE == 1
+  asm volatile("ld.global" GAR_LDH ".u16 %0, [%1];" : "=h"(v) : "l"(p));
+#elif GAR_DTYPE == 2
+  asm volatile("ld.global" GAR_LDH ".b32 %0, [%1];" : "=r"(v) : "l"(p));
+#else
+  asm volatile("ld.global" GAR_LDH ".f32 %0, [%1];" : "=f"(v) : "l"(p));
+#endif
+  return v;
+}
+static __device__ __forceinline__ void gar_stio(gar_io *p, gar_acc v) {
+#if GAR_DTYPE == 1
+  gar_u16 h;
+  asm("cvt.rn.bf16.f32 %0, %1;" : "=h"(h) : "f"(v));
+  asm volatile("st.global" GAR_STH ".u16 [%0], %1;" :: "l"(p), "h"(h) : "memory");
+#elif GAR_DTYPE == 2
+  asm volatile("st.global" GAR_STH ".b32 [%0], %1;" :: "l"(p), "r"(v) : "memory");
+#else
+  asm volatile("st.global" GAR_STH ".f32 [%0], %1;" :: "l"(p), "f"(v) : "memory");
+#endif
+}
+#if GAR_DTYPE == 1 && GAR_OP == 0
+// (widened bf16 h) + c with one rounding: the fp32 sum of the exactly widened value
+static __device__ __forceinline__ float gar_addbf(gar_u16 h, float c) {
+  float r;
+  asm("add.rn.f32.bf16 %0, %1, %2;" : "=f"(r) : "h"(h), "f"(c));
+  return r;
+}
+#endif
+)CUDA";
+
+}  // namespace
+
+int fused_peak_live(const gar_plan &pl) { return order_program(pl.prog).peak_live; }
+
+CodegenResult generate_fused_bf_source(const gar_plan &pl) {
+  const FusedProgram &fp = pl.prog;
+  const int P = pl.P;
+  const int nc = (int)fp.a.size();
+  const int nv = P + nc;
+  if ((int)fp.place.size() != nc || (int)fp.star.size() != nc)
+    throw std::logic_error("fused program without placements");
+  const bool rotate = pl.K != P;
+  const bool xr = pl.group == GAR_GROUP_XOR;
+  const bool sum_f = pl.op == GAR_SUM && pl.dtype != GAR_I32;
+  const bool bf16_sum = pl.op == GAR_SUM && pl.dtype == GAR_BF16;
+
+  // level of a value: the step that creates it (contributions: 0); combines by level
+  std::vector<int> level(nv, 0);
+  int maxlvl = 0;
+  for (int k = 0; k < nc; ++k) {
+    level[P + k] = 1 + std::max(level[fp.a[k]], level[fp.b[k]]);
+    maxlvl = std::max(maxlvl, level[P + k]);
+  }
+  // order of a level's combines: 0 as built (the q* of a step, then its q'), 1 by
+  // placement with q' first, 2 by placement with q* first (GAR_TUNE_BF_ORDER)
+  const int order = tune_int("GAR_TUNE_BF_ORDER", 2);
+  std::vector<std::vector<int>> comb(maxlvl + 1);
+  for (int k = 0; k < nc; ++k) comb[level[P + k]].push_back(k);
+  if (order != 0)
+    for (auto &cl : comb)
+      std::stable_sort(cl.begin(), cl.end(), [&](int x, int y) {
+        if (fp.place[x] != fp.place[y]) return fp.place[x] < fp.place[y];
+        return order == 1 ? fp.star[x] < fp.star[y] : fp.star[x] > fp.star[y];
+      });
+  std::vector<char> needs_leaf(P, 0);
+  for (int k = 0; k < nc; ++k)
+    for (int x : {fp.a[k], fp.b[k]})
+      if (x < P) needs_leaf[x] = 1;
+  for (int v : fp.out)
+    if (v < P) needs_leaf[v] = 1;
+
+  // Paired adds: combines (c1, c2) of one level whose operands are the low and high
+  // halves of pairs, in that order; their results become a pair.  Results at placements
+  // 2k and 2k + 1 of the same kind (q' or q*) also form a pair for later levels when
+  // they were computed one by one.  fp32 contributions pair as 2k, 2k + 1; bf16 ones go
+  // through the mixed add instead.
+  std::vector<int> pair_hi(nv, -1), mate(nc, -1);
+  std::vector<char> is_hi(nc, 0), hi_taken(nv, 0);
+  if (sum_f) {
+    std::map<std::pair<int, int>, int> by_ops;
+    for (int k = 0; k < nc; ++k) by_ops[{fp.a[k], fp.b[k]}] = k;
+    if (pl.dtype == GAR_F32)
+      for (int j = 0; j + 1 < P; j += 2) {
+        pair_hi[j] = j + 1;
+        hi_taken[j + 1] = 1;
+      }
+    for (int L = 1; L <= maxlvl; ++L) {
+      const std::vector<int> &cl = comb[L];
+      for (int c1 : cl) {
+        if (mate[c1] >= 0 || is_hi[c1]) continue;
+        const int ha = pair_hi[fp.a[c1]], hb = pair_hi[fp.b[c1]];
+        if (ha < 0 || hb < 0) continue;
+        auto it = by_ops.find({ha, hb});
+        if (it == by_ops.end()) continue;
+        const int c2 = it->second;
+        if (c2 == c1 || mate[c2] >= 0 || is_hi[c2] || level[P + c2] != L) continue;
+        mate[c1] = c2;
+        is_hi[c2] = 1;
+        pair_hi[P + c1] = P + c2;
+        hi_taken[P + c2] = 1;
+      }
+      std::map<std::pair<int, int>, int> at;  // (placement, star) -> value
+      for (int c : cl) at[{fp.place[c], fp.star[c]}] = P + c;
+      for (int c : cl) {
+        const int v = P + c;
+        if (fp.place[c] % 2 != 0 || pair_hi[v] >= 0 || is_hi[c]) continue;
+        auto it = at.find({fp.place[c] + 1, fp.star[c]});
+        if (it == at.end() || hi_taken[it->second] || pair_hi[it->second] >= 0) continue;
+        pair_hi[v] = it->second;
+        hi_taken[it->second] = 1;
+      }
+    }
+  }
+
+  // Launch shape, from P = 127 x 8 MiB bf16 on GB300: the widest programs (S = 7, 254
+  // live values) at 255 registers in 32-thread CTAs, 8 per SM (0.60 ms; 0.63 ms in
+  // 64-thread CTAs); the others at 168 registers (a third warp per sub-partition register
+  // file) in 64-thread CTAs (S = 8, 192 live values: 0.47 ms; 0.60 ms at 255 registers).
+  const int peak = order_program(fp).peak_live;
+  const bool widest = peak >= 224;
+  const int warps = std::max(1, std::min(16, tune_int("GAR_TUNE_BF_WARPS", widest ? 1 : 2)));
+  const int minb = std::max(1, tune_int("GAR_TUNE_BF_MINB", widest ? 8 : 5));
+  // Pointer tables: the kernel parameters, indexed b + j (stored twice), while a warp's
+  // 32 element positions share one block almost always (blocks of 32+ elements); with
+  // shorter blocks the index differs across the lanes and the tables go to shared memory.
+  const bool smem_tab = rotate && pl.n / (uint64_t)P < 32;
+  const int tp = (rotate && !xr) ? 2 * P : P;
+  CodegenResult cg;
+  cg.width = 1;
+  cg.table_copies = (rotate && !xr) ? 2 : 1;
+  cg.threads = 32 * warps;
+  cg.form = 1;
+  cg.kernel_name = fmt("gar_fusedbf_P%d_S%d_K%d_", P, pl.S, pl.K) + dtype_tag(pl.dtype) + "_" +
+                   op_tag(pl.op) + (xr ? "_xor" : "");
+
+  std::string s;
+  s += fmt("#define GAR_DTYPE %d\n#define GAR_OP %d\n", pl.dtype, pl.op);
+  s += "#define GAR_LDH \"" + tune_str("GAR_TUNE_LDH", ".cs") + "\"\n";
+  s += "#define GAR_STH \"" + tune_str("GAR_TUNE_STH", ".cs") + "\"\n";
+  s += kSkeleton;
+  s += kBFHelpers;
+  s += fmt("struct gar_args { const gar_io *in[%d]; gar_io *out[%d]; gar_u64 e_lo, e_hi; };\n",
+           cg.table_copies * P, cg.table_copies * P);
+  if (rotate) s += emit_block_of("gar_block_of", P, pl.n);
+
+  // contribution j of an element of block b comes from rank t_j(b); result placement p
+  // goes to rank t_p(b) (latency-optimal programs: no rotation, b = 0)
+  auto rank_of = [&](int j) -> std::string {
+    if (!rotate) return std::to_string(j);
+    if (j == 0) return "b";
+    return xr ? fmt("(b ^ %d)", j) : fmt("(b + %d)", j);
+  };
+  const std::string tin = smem_tab ? "tin[" : "a.in[", tout = smem_tab ? "tout[" : "a.out[";
+  std::string f = "static __device__ __forceinline__ void gar_eval_bf(const gar_args &a, ";
+  f += smem_tab ? "const gar_io *const *tin, gar_io *const *tout, " : "";
+  f += "gar_u64 e, int b) {\n  (void)a; (void)b;\n";
+  for (int j = 0; j < P; ++j)
+    if (needs_leaf[j]) f += fmt("  const gar_io l%d = gar_ldio(", j) + tin + rank_of(j) + "] + e);\n";
+  auto opnd = [&](int x) { return x < P ? fmt("gar_wide(l%d)", x) : fmt("v%d", x); };
+  for (int L = 1; L <= maxlvl; ++L) {
+    for (int k : comb[L]) {
+      if (is_hi[k]) continue;
+      const int v = P + k, a = fp.a[k], b = fp.b[k];
+      if (mate[k] >= 0) {
+        const int k2 = mate[k], v2 = P + k2;
+        f += fmt("  const float2 w%d = __fadd2_rn(make_float2(", v) + opnd(a) + ", " + opnd(fp.a[k2]) +
+             "), make_float2(" + opnd(b) + ", " + opnd(fp.b[k2]) + "));\n";
+        f += fmt("  const gar_acc v%d = w%d.x, v%d = w%d.y;\n", v, v, v2, v);
+      } else if (bf16_sum && (a < P || b < P)) {
+        const int lf = a < P ? a : b, other = a < P ? b : a;
+        f += fmt("  const gar_acc v%d = gar_addbf(l%d, ", v, lf) + opnd(other) + ");\n";
+      } else {
+        f += fmt("  const gar_acc v%d = gar_op(", v) + opnd(a) + ", " + opnd(b) + ");\n";
+      }
+    }
+  }
+  std::vector<std::vector<int>> places_of(fp.K);
+  for (int p = 0; p < P; ++p) places_of[fp.origin[p]].push_back(p);
+  for (int sc = 0; sc < fp.K; ++sc)
+    for (int p : places_of[sc]) f += "  gar_stio(" + tout + rank_of(p) + "] + e, " + opnd(fp.out[sc]) + ");\n";
+  f += "}\n";
+  s += f;
+
+  s += fmt("extern \"C\" __global__ void __launch_bounds__(%d, %d) ", cg.threads, minb) + cg.kernel_name +
+       "(const __grid_constant__ gar_args a) {\n";
+  if (smem_tab) {
+    s += fmt("  __shared__ const gar_io *s_in[%d];\n  __shared__ gar_io *s_out[%d];\n", tp, tp);
+    s += fmt("  for (int i = threadIdx.x; i < %d; i += blockDim.x) { s_in[i] = a.in[i]; s_out[i] = a.out[i]; }\n", tp);
+    s += "  __syncthreads();\n";
+  }
+  // launched with programmatic stream serialisation: nothing is read before every
+  // earlier kernel on the stream has completed
+  s += "  asm volatile(\"griddepcontrol.wait;\" ::: \"memory\");\n";
+  s += "  const gar_u64 npos = a.e_hi - a.e_lo;\n";
+  s += "  const gar_u64 stride = (gar_u64)gridDim.x * blockDim.x;\n";
+  // one element position per thread
+  s += "  for (gar_u64 i = (gar_u64)blockIdx.x * blockDim.x + threadIdx.x; i < npos; i += stride) {\n";
+  s += "    const gar_u64 e = a.e_lo + i;\n";
+  s += rotate ? "    const int b = gar_block_of(e);\n" : "    const int b = 0;\n";
+  s += std::string("    gar_eval_bf(a, ") + (smem_tab ? "s_in, s_out, " : "") + "e, b);\n";
+  s += "  }\n";
+  s += "  asm volatile(\"griddepcontrol.launch_dependents;\" ::: \"memory\");\n}\n";
+  cg.source = s;
+  return cg;
+}
+
 
 CodegenResult generate_batched_source(const std::vector<const gar_plan *> &plans) {
   const gar_plan &p0 = *plans[0];

@@ -66,6 +66,8 @@ struct CommStep {
 struct FusedProgram {
   int P = 0, K = 0;
   std::vector<int32_t> a, b;      // combine k: value P + k = a[k] (+) b[k]
+  std::vector<int32_t> place;     // combine k: placement its result lives at (contribution j: j)
+  std::vector<int8_t> star;       // combine k: 1 if its result is a q* vector, 0 if a q' vector
   std::vector<int32_t> out;       // out[s] = value id of result copy s
   std::vector<int32_t> origin;    // origin[p] = copy written to placement p
 };
@@ -132,8 +134,14 @@ struct CodegenResult {
   std::string kernel_name;
   int width = 1;
   int table_copies = 1;  // fused kernels: copies of the in[] / out[] pointer tables (1 or 2)
+  int threads = 256;     // threads per CTA
+  int form = 0;          // fused kernels: 0 single-thread program, 1 breadth-first
 };
 CodegenResult generate_fused_source(const gar_plan &pl);
+// The breadth-first form of the fused kernel (programs with many result copies), and
+// the peak number of live values of a plan's program in the single-thread form.
+CodegenResult generate_fused_bf_source(const gar_plan &pl);
+int fused_peak_live(const gar_plan &pl);
 CodegenResult generate_batched_source(const std::vector<const gar_plan *> &plans);
 
 // jit.cpp
@@ -145,6 +153,7 @@ struct JitKernel {
   int width = 1;
   int table_copies = 1;
   int threads = 256;
+  int form = 0;
   int blocks_per_sm = 0;
   int regs = 0, local_bytes = 0;
   bool loaded = false;

@@ -59,6 +59,8 @@ int jit_compile(const CodegenResult &cg, JitKernel **out) {
   k->name = cg.kernel_name;
   k->width = cg.width;
   k->table_copies = cg.table_copies;
+  k->threads = cg.threads;
+  k->form = cg.form;
   *out = k.get();
   g_cache.emplace(cg.source, std::move(k));
   return GAR_OK;

@@ -255,15 +255,21 @@ void build_fused(gar_plan *pl) {
   fp.P = P;
   fp.K = K;
   std::map<std::pair<int, int>, int> cse;
-  std::vector<int32_t> A, B;
-  auto mk = [&](int a, int b) {
+  std::vector<int32_t> A, B, PL;
+  std::vector<int8_t> ST;
+  auto mk = [&](int a, int b, int place, int star) {
     if (a < 0 || b < 0) throw std::logic_error("fused program reads a dead vector");
     auto key = std::make_pair(a, b);
     auto it = cse.find(key);
-    if (it != cse.end()) return it->second;
+    if (it != cse.end()) {
+      if (PL[it->second - P] != place) throw std::logic_error("one vector at two placements");
+      return it->second;
+    }
     const int id = P + (int)A.size();
     A.push_back(a);
     B.push_back(b);
+    PL.push_back(place);
+    ST.push_back((int8_t)star);
     cse.emplace(key, id);
     return id;
   };
@@ -276,9 +282,9 @@ void build_fused(gar_plan *pl) {
     std::vector<int> nqp(P, -1), nqs(K);
     // q*_s first, then q'_p: the values are CSE'd, the order only fixes numbering
     // the vector received at placement p came from placement t_d(p)
-    for (int s = 0; s < K; ++s) nqs[s] = even ? mk(qs[s], qp[g.op(s, d)]) : qs[s];
+    for (int s = 0; s < K; ++s) nqs[s] = even ? mk(qs[s], qp[g.op(s, d)], s, 1) : qs[s];
     if (c >= 2)
-      for (int32_t p : union_placements(g, K, 1, c - 1)) nqp[p] = mk(qp[p], qp[g.op(p, d)]);
+      for (int32_t p : union_placements(g, K, 1, c - 1)) nqp[p] = mk(qp[p], qp[g.op(p, d)], p, 0);
     qp.swap(nqp);
     qs.swap(nqs);
   }
@@ -303,6 +309,8 @@ void build_fused(gar_plan *pl) {
     renum[P + k] = P + (int)fp.a.size();
     fp.a.push_back(renum[A[k]]);
     fp.b.push_back(renum[B[k]]);
+    fp.place.push_back(PL[k]);
+    fp.star.push_back(ST[k]);
   }
   for (int s = 0; s < K; ++s) fp.out.push_back(renum[qs[s]]);
   // Origins: copy s sits at placement s; distribution step i (reversed) copies
@@ -416,6 +424,8 @@ void build_folds(gar_plan *pl) {
     for (int k = N - 2 * f; k < N - f; ++k) {
       fp.a.push_back(qp[k]);
       fp.b.push_back(qp[k + f]);
+      fp.place.push_back(k);
+      fp.star.push_back(0);
       qp[k] = P + (int)fp.a.size() - 1;
     }
   }
@@ -489,6 +499,8 @@ void build_ring(gar_plan *pl) {
   for (int k = 1; k < P; ++k) {
     fp.a.push_back(k);
     fp.b.push_back(v);
+    fp.place.push_back(k);
+    fp.star.push_back(0);
     v = P + (int)fp.a.size() - 1;
   }
   fp.out.push_back(v);

@@ -1,0 +1,211 @@
+"""Host-side checks of the breadth-first fused kernel (no GPU).
+
+The breadth-first form evaluates a plan's combine program step by step, with paired
+fp32 adds and bf16 mixed adds.  These tests check, without a GPU:
+  * which plans take it (gar_plan_info.fused_form);
+  * that its generated evaluation code, run by a small interpreter written here in
+    numpy float32, gives the oracle's bits for every rank and element, at every step
+    count, for cyclic and XOR groups, sums and max/min, and rotated block layouts;
+  * that NVRTC compiles it for sm_103a for a range of plans.
+"""
+
+import os
+import re
+
+import numpy as np
+import pytest
+
+from oracle import gar_oracle as O
+from paper_2004_09362_gb300 import gar as G
+
+
+def _with_form(form, fn):
+    old = os.environ.get("GAR_TUNE_FUSED_FORM")
+    os.environ["GAR_TUNE_FUSED_FORM"] = str(form)
+    try:
+        return fn()
+    finally:
+        if old is None:
+            os.environ.pop("GAR_TUNE_FUSED_FORM", None)
+        else:
+            os.environ["GAR_TUNE_FUSED_FORM"] = old
+
+
+def _bf_source(P, n, dtype, S, op="sum", group="cyclic"):
+    def make():
+        pl = G.gar_plan_create_group(P, n, dtype, op, S, group)
+        return G.gar_plan_fused_source(pl), G.gar_plan_get_info(pl)
+    return _with_form(1, make)
+
+
+# ---------------------------------------------------------------------------
+# Which plans take the breadth-first form
+# ---------------------------------------------------------------------------
+
+def test_selection():
+    form = {S: G.gar_plan_get_info(G.gar_plan_create(127, 4194304, "bf16", "sum", S))["fused_form"]
+            for S in range(7, 15)}
+    assert form == {7: 1, 8: 1, 9: 0, 10: 0, 11: 0, 12: 0, 13: 0, 14: 0}
+    assert G.gar_plan_get_info(G.gar_plan_create(127, 4096, "f32", "sum", 7))["fused_form"] == 1
+    for dtype, op in (("bf16", "max"), ("f32", "min"), ("i32", "sum")):
+        assert G.gar_plan_get_info(G.gar_plan_create(127, 4096, dtype, op, 7))["fused_form"] == 0
+    for P, S in ((24, 10), (64, 6), (8, 3), (5, 3)):
+        assert G.gar_plan_get_info(G.gar_plan_create(P, 4096, "f32", "sum", S))["fused_form"] == 0
+
+
+def test_every_combine_emitted_once():
+    """P = 127, S = 7: the 1524 combines are 2 x (paired adds) + single adds, and the
+    even-distance steps pair most of them."""
+    src, info = _bf_source(127, 4194304, "bf16", 7)
+    pairs = src.count("__fadd2_rn(make_float2(")
+    singles = len(re.findall(r"const gar_acc v\d+ = gar_(?:addbf|op)\(", src))
+    assert 2 * pairs + singles == info["fused_combines"] == 1524
+    assert pairs >= 500
+    assert "__launch_bounds__(32, 8)" in src      # 254 live values: 255 registers
+    src8, _ = _bf_source(127, 4194304, "bf16", 8)
+    assert "__launch_bounds__(64, 5)" in src8     # 192 live values: 168 registers
+
+
+# ---------------------------------------------------------------------------
+# Interpreter of the generated evaluation function
+# ---------------------------------------------------------------------------
+
+def _bf16_round(x):
+    return O.round_to_bf16(np.asarray(x, dtype=np.float32))
+
+
+def _run_generated(src, P, xs, dtype, op):
+    """Evaluates gar_eval_bf for every element e of P rank vectors xs (numpy), returning
+    the P output vectors.  The interpreter knows the few statement forms the generator
+    emits; rank expressions are evaluated with the element's block b (mod P for the
+    doubled pointer tables)."""
+    body = re.search(r"void gar_eval_bf\(.*?\{\n(.*?)\n\}\n", src, re.S).group(1)
+    n = len(xs[0])
+    nblk = re.search(r"return e < big \? \(int\)\(e / (\d+)ULL\) : \(int\)\((\d+)ULL \+ \(e - big\) / (\d+)ULL\)", src)
+    bigm = re.search(r"const gar_u64 big = (\d+)ULL;", src)
+
+    def block_of(e):
+        if "gar_block_of" not in src:
+            return 0
+        if nblk is None:
+            return e
+        q1, rem, q = int(nblk.group(1)), int(nblk.group(2)), int(nblk.group(3))
+        big = int(bigm.group(1))
+        return e // q1 if e < big else rem + (e - big) // q
+
+    xor = "(b ^" in body
+
+    def rank(expr, b):
+        expr = expr.strip()
+        val = eval(expr, {}, {"b": b})  # generated arithmetic on b only
+        return val % P if not xor else val
+
+    comb = {"sum": lambda a, c: np.float32(a + c), "max": lambda a, c: np.float32(max(a, c)),
+            "min": lambda a, c: np.float32(min(a, c))}[op]
+    if dtype == "i32":
+        comb = {"sum": lambda a, c: np.int32((int(a) + int(c) + 2**31) % 2**32 - 2**31),
+                "max": lambda a, c: max(a, c), "min": lambda a, c: min(a, c)}[op]
+    out = [np.zeros_like(x) for x in xs]
+    lines = [ln.strip() for ln in body.split("\n") if ln.strip() and not ln.strip().startswith("(void)")]
+    for e in range(n):
+        b = block_of(e)
+        env = {}
+
+        def val(tok):
+            tok = tok.strip()
+            m = re.fullmatch(r"gar_wide\((l\d+)\)", tok)
+            return env[m.group(1)] if m else env[tok]
+
+        for ln in lines:
+            m = re.fullmatch(r"const gar_io (l\d+) = gar_ldio\((?:a\.in|tin)\[(.*)\] \+ e\);", ln)
+            if m:
+                env[m.group(1)] = xs[rank(m.group(2), b)][e]
+                continue
+            m = re.fullmatch(r"const float2 (w\d+) = __fadd2_rn\(make_float2\((.*), (.*)\), make_float2\((.*), (.*)\)\);", ln)
+            if m:
+                env[m.group(1)] = (np.float32(val(m.group(2)) + val(m.group(4))),
+                                   np.float32(val(m.group(3)) + val(m.group(5))))
+                continue
+            m = re.fullmatch(r"const gar_acc (v\d+) = (w\d+)\.x, (v\d+) = \2\.y;", ln)
+            if m:
+                env[m.group(1)], env[m.group(3)] = env[m.group(2)]
+                continue
+            m = re.fullmatch(r"const gar_acc (v\d+) = gar_addbf\((l\d+), (.*)\);", ln)
+            if m:
+                env[m.group(1)] = np.float32(env[m.group(2)] + val(m.group(3)))
+                continue
+            m = re.fullmatch(r"const gar_acc (v\d+) = gar_op\((.*), (.*)\);", ln)
+            if m:
+                env[m.group(1)] = comb(val(m.group(2)), val(m.group(3)))
+                continue
+            m = re.fullmatch(r"gar_stio\((?:a\.out|tout)\[(.*)\] \+ e, (.*)\);", ln)
+            if m:
+                v = val(m.group(2))
+                out[rank(m.group(1), b)][e] = _bf16_round(np.float32([v]))[0] if dtype == "bf16" else v
+                continue
+            raise AssertionError("statement the interpreter does not know: " + ln)
+    return out
+
+
+def _inputs(P, n, dtype, seed):
+    rng = np.random.default_rng(seed)
+    if dtype == "i32":
+        return [rng.integers(-1000, 1000, n).astype(np.int32) for _ in range(P)]
+    xs = [(rng.standard_normal(n) * np.exp2(rng.integers(-12, 13, n))).astype(np.float32) for _ in range(P)]
+    return [_bf16_round(x) for x in xs] if dtype == "bf16" else xs
+
+
+CASES = ([(P, "f32", "sum", "cyclic") for P in (3, 5, 6, 7, 9, 12, 13)] +
+         [(7, "bf16", "sum", "cyclic"), (11, "bf16", "sum", "cyclic"), (6, "f32", "max", "cyclic"),
+          (5, "i32", "min", "cyclic"), (8, "f32", "sum", "xor"), (16, "bf16", "sum", "xor")])
+
+
+@pytest.mark.parametrize("P,dtype,op,group", CASES)
+def test_generated_code_reproduces_oracle(P, dtype, op, group):
+    """Bit for bit against the oracle at every step count in [L, 2L] with more than one
+    result copy, with n = 3P + 2 (ragged blocks, every rotation b)."""
+    n = 3 * P + 2
+    xs = _inputs(P, n, dtype, seed=P * 31 + len(dtype))
+    L = max(1, (P - 1).bit_length())
+    for S in range(L, 2 * L):
+        src, info = _bf_source(P, n, dtype, S, op, group)
+        assert info["K"] > 1
+        got = _run_generated(src, P, xs, dtype, op)
+        want = O.allreduce(xs, S, op, dtype, group=group)
+        for x in range(P):
+            np.testing.assert_array_equal(np.asarray(got[x]).view(np.uint32 if dtype != "i32" else np.int32),
+                                          np.asarray(want[x], dtype=got[x].dtype).view(np.uint32 if dtype != "i32" else np.int32),
+                                          err_msg=f"P={P} S={S} rank {x}")
+
+
+def test_interpreter_catches_a_planted_mistake():
+    """The interpreter is not vacuous: swapping two result stores in the generated text
+    breaks the comparison."""
+    P, n, S = 7, 23, 3
+    xs = _inputs(P, n, "f32", 5)
+    src, _ = _bf_source(P, n, "f32", S)
+    stores = re.findall(r"gar_stio\(a\.out\[(\d+)\] \+ e, (v\d+)\);", src)
+    (r0, v0), (r1, v1) = stores[0], stores[1]
+    bad = src.replace(f"a.out[{r0}] + e, {v0});", "@@").replace(f"a.out[{r1}] + e, {v1});", f"a.out[{r1}] + e, {v0});")
+    bad = bad.replace("@@", f"a.out[{r0}] + e, {v1});")
+    assert bad != src
+    got = _run_generated(bad, P, xs, "f32", "sum")
+    want = O.allreduce(xs, S, "sum", "f32")
+    assert any(not np.array_equal(got[x], want[x]) for x in range(P))
+
+
+# ---------------------------------------------------------------------------
+# NVRTC compiles the form (host only)
+# ---------------------------------------------------------------------------
+
+@pytest.mark.parametrize("P", [2, 3, 5, 8, 12, 24, 33])
+def test_breadth_first_kernels_compile(P):
+    def go():
+        L = max(1, (P - 1).bit_length())
+        for dtype in ("f32", "bf16", "i32"):
+            for op in ("sum", "max"):
+                for S in range(L, 2 * L + 1):
+                    G.gar_plan_compile(G.gar_plan_create(P, 4 * P + 3, dtype, op, S), "fused")
+        if P & (P - 1) == 0:
+            G.gar_plan_compile(G.gar_plan_create_group(P, 1000, "f32", "sum", L, "xor"), "fused")
+    _with_form(1, go)

@@ -243,6 +243,38 @@ def test_latency_optimal_mid_size_fused(P, n, dtype):
 
 
 # ---------------------------------------------------------------------------
+# The breadth-first fused form (step by step, paired fp32 adds, bf16 mixed adds)
+# ---------------------------------------------------------------------------
+
+@pytest.mark.parametrize("P,n", [(40, 40 * 97 + 13), (127, 127 * 40 + 19), (127, 3 * 127 + 5)])
+@pytest.mark.parametrize("dtype,op", [("f32", "sum"), ("bf16", "sum"), ("i32", "sum"), ("f32", "max")])
+def test_breadth_first_form_every_step_count(P, n, dtype, op, monkeypatch):
+    """The breadth-first form forced on for every step count with several result copies
+    (it is the default only for large float sums at small S), bit for bit against the
+    oracle; n = 3P + 5 puts several blocks in one warp (pointer tables in shared memory)."""
+    monkeypatch.setenv("GAR_TUNE_FUSED_FORM", "1")
+    t = _np_inputs(P, n, dtype, seed=P + n)
+    host = _to_host_list(t, dtype)
+    L = G.ceil_log2(P)
+    for S in range(L, 2 * L):
+        plan = gar.gar_plan_create(P, n, dtype, op, S)
+        assert gar.gar_plan_get_info(plan)["fused_form"] == gar.GAR_FORM_BREADTH
+        _assert_same(_run(plan, t, "fused"), G.allreduce(host, S, op, dtype), dtype, f"S={S}")
+
+
+@pytest.mark.parametrize("P", [8, 32])
+def test_breadth_first_form_xor_group(P, monkeypatch):
+    monkeypatch.setenv("GAR_TUNE_FUSED_FORM", "1")
+    n = 5 * P + 3
+    t = _np_inputs(P, n, "f32", seed=P)
+    host = _to_host_list(t, "f32")
+    L = G.ceil_log2(P)
+    for S in range(L, 2 * L):
+        plan = gar.gar_plan_create_group(P, n, "f32", "sum", S, "xor")
+        _assert_same(_run(plan, t, "fused"), G.allreduce(host, S, "sum", "f32", group="xor"), "f32", f"S={S}")
+
+
+# ---------------------------------------------------------------------------
 # Recorded step bytes equal the schedule's predicted volume
 # ---------------------------------------------------------------------------
 
