@@ -179,12 +179,17 @@ def _time_loop(fn, steps, warmup, stream, flush=None):
 
 
 class L2Flusher:
+    """Evicts L2 (129 MB on GB300) by reading a 512 MiB buffer into a scalar.  A read
+    leaves only clean lines in L2, so nothing is written back inside the timed call that
+    follows; the dirty lines of the previous call are written back during the flush."""
+
     def __init__(self, nbytes=512 << 20):
         import torch
-        self.buf = torch.empty(nbytes // 4, dtype=torch.int32, device="cuda")
+        self.buf = torch.zeros(nbytes // 4, dtype=torch.int32, device="cuda")
+        self.acc = torch.int64
 
     def __call__(self):
-        self.buf.add_(1)
+        self.buf.sum(dtype=self.acc)
 
 
 # ---------------------------------------------------------------------------
@@ -273,12 +278,12 @@ def run_ours(args):
         dtype = wl.dtype
         inp = gar_inputs.rank_inputs(P, n, wl.dtype, wl.dist, wl.seed + rank, device="cuda")
         plan = gar.gar_plan_create(P, n, wl.dtype, args.op, S)
-        if args.mode == "step":
+        if args.mode in ("step", "persistent"):
             gar.ensure_workspace(plan)
         gar.gar_plan_prepare(plan, args.mode)
         ptrs = gar.rank_pointers(inp)
         info = plan.info()
-        launches_per_step = 1 if args.mode == "fused" else info["n_launches"]
+        launches_per_step = 1 if args.mode in ("fused", "persistent") else info["n_launches"]
         if args.mode == "fused":
             bytes_step = _alg_bytes(P, n, wl.dtype)
         else:
@@ -305,7 +310,7 @@ def run_ours(args):
     with ClockSampler(local) as clk:
         # untimed load window of the same step, so the clock samples (every 100 ms)
         # see the GPU under this load; the timed region follows without a pause
-        t_end = time.time() + CLOCK_WINDOW_S
+        t_end = time.time() + args.clock_window
         while time.time() < t_end:
             for _ in range(8):
                 step()
@@ -328,7 +333,7 @@ def run_ours(args):
     else:
         value = job_gbs(_alg_bytes(P, n, dtype), ws, ms)
     clocks = clk.summary()
-    clocks["window"] = (f"{CLOCK_WINDOW_S:.1f} s of untimed steps right before the timed "
+    clocks["window"] = (f"{args.clock_window:.1f} s of untimed steps right before the timed "
                         f"{args.steps}, sampled every 100 ms through both")
     kernel_gbs = bytes_step / (ms * 1e-3) / 1e9
 
@@ -398,6 +403,31 @@ def _committed_traffic(gar):
         return None
 
 
+def _link_ceiling(host_in, host_out, dev_dst, dev_src, reps=3):
+    """GB/s of the host link with both directions busy: host_in -> dev_dst and dev_src ->
+    host_out (pinned, one copy each) on two streams at once; best of `reps`."""
+    import torch
+    s1, s2 = torch.cuda.Stream(), torch.cuda.Stream()
+    nbytes = host_in.numel() * host_in.element_size() + dev_src.numel() * dev_src.element_size()
+    best = None
+    for _ in range(reps):
+        torch.cuda.synchronize()
+        start, mid, end = (torch.cuda.Event(enable_timing=True) for _ in range(3))
+        start.record(s1)
+        s2.wait_event(start)
+        with torch.cuda.stream(s1):
+            dev_dst.copy_(host_in, non_blocking=True)
+        with torch.cuda.stream(s2):
+            host_out.copy_(dev_src, non_blocking=True)
+        mid.record(s2)
+        s1.wait_event(mid)
+        end.record(s1)
+        torch.cuda.synchronize()
+        ms = start.elapsed_time(end)
+        best = ms if best is None else min(best, ms)
+    return nbytes / (best * 1e-3) / 1e9
+
+
 def _e2e(gar, plan, inp, P, n, dtype, args, stream, dist):
     import torch
     host_in = inp.cpu().pin_memory()
@@ -416,9 +446,14 @@ def _e2e(gar, plan, inp, P, n, dtype, args, stream, dist):
     ms = max_over_ranks(_time_loop(step, steps, 3, stream), dist, "cuda")
     ws = dist.get_world_size() if dist is not None else 1
     bytes_step = _alg_bytes(P, n, dtype)
-    return {"value": round(job_gbs(bytes_step, ws, ms), 2), "unit": "GB/s",
+    value = job_gbs(bytes_step, ws, ms)
+    link = _link_ceiling(host_in, host_out, dev, inp)
+    return {"value": round(value, 2), "unit": "GB/s",
             "ms_per_step": round(ms, 4), "h2d_bytes_per_step": bytes_step // 2,
             "d2h_bytes_per_step": bytes_step // 2, "steps": steps,
+            "link_ceiling_gbs": round(link, 1), "frac_of_link": round(value / ws / link, 4),
+            "link_ceiling": ("the same bytes moved by one cudaMemcpyAsync host-to-device and one "
+                             "device-to-host, pinned memory, on two streams at once (best of 3, same run)"),
             "path": ("gar_allreduce_host on pinned host buffers: the fused kernel reads the P inputs "
                      "from and writes the P results to host memory over NVLink-C2C (no staging copies)")
             if args.mode == "fused" else
@@ -467,7 +502,8 @@ def measure_rows(gar, gar_inputs, stream, hbm_peak):
                "fused_GB/s": round(_alg_bytes(P, n, "bf16") / ms_f / 1e6, 1),
                "fused_frac": round(_alg_bytes(P, n, "bf16") / ms_f / 1e6 / hbm_peak, 4),
                "fused_combines_per_position": plan.info()["fused_combines"],
-               "fused_width": plan.info()["fused_width"]}
+               "fused_width": plan.info()["fused_width"],
+               "fused_form": "breadth_first" if plan.info()["fused_form"] == 1 else "single"}
         if S in (7, 10, 14):
             gar.ensure_workspace(plan)
             ms_s = _time_loop(lambda: gar.gar_allreduce(plan, inp, "step", stream), 2, 1, stream)
@@ -483,7 +519,7 @@ def measure_rows(gar, gar_inputs, stream, hbm_peak):
     rows["p127_8mib_bf16"] = sweep
     del inp
 
-    # P=8, 1 MiB per rank: L2-resident, so flush L2 before each call
+    # P=8, 1 MiB per rank: L2-resident, so flush L2 (read-only sweep) before each call
     wl = gar_inputs.WORKLOADS["p8_1mib_f32"]
     P, n = wl.P, wl.n
     inp = gar_inputs.rank_inputs(P, n, wl.dtype, wl.dist, wl.seed, device="cuda")
@@ -537,7 +573,7 @@ def measure_rows(gar, gar_inputs, stream, hbm_peak):
     torch.cuda.empty_cache()
     rows["groups_p64_4mib_f32"] = groups_row(gar, gar_inputs, stream, hbm_peak)
     rows["step_range_p24_64mib_f32"] = step_range_row(gar, gar_inputs, stream, hbm_peak)
-    rows["cost_model_p127_bf16_step"] = cost_model_row(gar, gar_inputs, stream)
+    rows["cost_model_p127_bf16_step"] = cost_model_row(gar, gar_inputs, stream, hbm_peak)
     return rows
 
 
@@ -605,7 +641,7 @@ def _paper_blocks(P, S):
     return 2 * (P - 1) + extra * (L - 1), (P - 1) + extra * (2 * L - 2)
 
 
-def cost_model_row(gar, gar_inputs, stream, P=127, dtype="bf16",
+def cost_model_row(gar, gar_inputs, stream, hbm_peak, P=127, dtype="bf16",
                    sizes=(425, 9 * 1024, 64 * 1024, 512 * 1024, 4 << 20, 8 << 20)):
     """Step-faithful mode as the paper's machine: measure every step count at several
     message sizes, fit the cost model's alpha (per step), beta (per byte moved) and gamma
@@ -645,21 +681,43 @@ def cost_model_row(gar, gar_inputs, stream, P=127, dtype="bf16",
         A.append([S / t, tr * u / t, co * u / t])
         y.append(1.0)
     coef, _res = nnls(np.array(A), np.array(y))
-    alpha, beta, gamma = (float(c) for c in coef)
-    per = {}
-    agree = 0
-    for m in sizes:
-        meas = {S: times[(m, S)] for S in range(L, 2 * L + 1)}
-        best_meas = min(meas, key=meas.get)
-        best_model = gar.gar_optimal_steps(P, m, alpha, beta, gamma)
-        agree += int(best_meas == best_model)
-        per[str(m)] = {"measured_us": {f"S{S}": round(t * 1e6, 2) for S, t in meas.items()},
-                       "model_us": {f"S{S}": round(gar.gar_cost_model(P, S, m, alpha, beta, gamma) * 1e6, 2)
-                                    for S in meas},
-                       "measured_best_S": best_meas, "model_best_S": best_model,
-                       "model_choice_vs_best": round(meas[best_model] / meas[best_meas], 3)}
-    return {"P": P, "dtype": dtype, "mode": "step", "alpha_s": alpha, "beta_s_per_B": beta,
-            "gamma_s_per_B": gamma, "argmin_agreement": f"{agree}/{len(sizes)}", "per_size_bytes": per}
+    fitted = tuple(float(c) for c in coef)
+    # Derived model: alpha = per-step time at the smallest size (slope of t over S);
+    # beta, gamma from the step kernels' DRAM traffic at the measured copy bandwidth --
+    # every byte of a block sent is one partner read, every byte combined one own read
+    # and one write, and all P ranks share one HBM, so a per-rank byte costs P bytes of
+    # DRAM time.
+    Ss = np.arange(L, 2 * L + 1, dtype=float)
+    ts = np.array([times[(sizes[0], int(S))] for S in Ss])
+    alpha_d = float(np.polyfit(Ss, ts, 1)[0])
+    bw = hbm_peak * 1e9
+    derived = (alpha_d, P / bw, 2 * P / bw)
+
+    def evaluate(a, b, g):
+        per, agree, worst = {}, 0, 1.0
+        for m in sizes:
+            meas = {S: times[(m, S)] for S in range(L, 2 * L + 1)}
+            best_meas = min(meas, key=meas.get)
+            best_model = gar.gar_optimal_steps(P, m, a, b, g)
+            agree += int(best_meas == best_model)
+            worst = max(worst, meas[best_model] / meas[best_meas])
+            per[str(m)] = {"model_us": {f"S{S}": round(gar.gar_cost_model(P, S, m, a, b, g) * 1e6, 2)
+                                        for S in meas},
+                           "measured_best_S": best_meas, "model_best_S": best_model,
+                           "model_choice_vs_best": round(meas[best_model] / meas[best_meas], 3)}
+        return {"alpha_s": a, "beta_s_per_B": b, "gamma_s_per_B": g,
+                "argmin_agreement": f"{agree}/{len(sizes)}", "worst_choice_vs_best": round(worst, 3),
+                "per_size_bytes": per}
+
+    measured = {str(m): {f"S{S}": round(times[(m, S)] * 1e6, 2) for S in range(L, 2 * L + 1)}
+                for m in sizes}
+    per_step_us = {str(m): {f"S{S}": round(times[(m, S)] * 1e6 / S, 2) for S in range(L, 2 * L + 1)}
+                   for m in sizes}
+    return {"P": P, "dtype": dtype, "mode": "step", "measured_us": measured,
+            "measured_us_per_step": per_step_us,
+            "fit_free": evaluate(*fitted), "fit_derived": evaluate(*derived),
+            "derived_from": f"alpha: slope of time over S at {sizes[0]} B; beta = P / HBM, "
+                            f"gamma = 2P / HBM with HBM = {hbm_peak} GB/s (measured copy)"}
 
 
 # ---------------------------------------------------------------------------
@@ -776,8 +834,11 @@ def main():
     ap.add_argument("--workload", default=HEADLINE,
                     help="gar_inputs.WORKLOADS key or batched_425B (default: the headline)")
     ap.add_argument("--S", type=int, default=None, help="step count (default: 2*ceil(log2 P))")
-    ap.add_argument("--mode", default="fused", choices=["fused", "step"])
+    ap.add_argument("--mode", default="fused", choices=["fused", "step", "persistent"])
     ap.add_argument("--op", default="sum", choices=["sum", "max", "min"])
+    ap.add_argument("--clock-window", type=float, default=CLOCK_WINDOW_S,
+                    help="seconds of untimed steps sampled for clocks before the timed region "
+                         "(0 for profiling runs: fewer launches before the captured ones)")
     args = ap.parse_args()
     if args.warmup < 3:
         args.warmup = 3

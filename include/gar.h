@@ -161,7 +161,8 @@ GAR_API int gar_plan_create_group(gar_plan **out, int P, uint64_t n, int dtype, 
                                   int group);
 
 /* Frees the plan and its device tables.  NULL is a no-op.  The caller must make sure
- * no work using the plan is still running. */
+ * no work using the plan is still running.  (Resource management; no counterpart in the
+ * paper.) */
 GAR_API void gar_plan_destroy(gar_plan *plan);
 
 /* Fills *info (see gar_plan_info).  Host-only. */
@@ -208,7 +209,10 @@ GAR_API int gar_plan_step_ops(const gar_plan *plan, int32_t *ops, int *nops, int
                       int *nlaunch);
 
 /* Caller-owned device workspace for step-faithful mode (16-byte aligned, at least
- * workspace_bytes).  NULL with 0 bytes detaches it. */
+ * workspace_bytes): the storage of the partial vectors q' and q* that the paper's
+ * processes keep between steps (Sec. "Latency-optimal version" keeps the two apart).
+ * The memory model has no counterpart in the paper.  NULL with 0 bytes detaches it.
+ * GAR_EALIGN for a misaligned pointer. */
 GAR_API int gar_plan_set_workspace(gar_plan *plan, void *dev_ptr, size_t bytes);
 
 /* The CUDA C source of the plan's generated fused kernel (host-only).  Copies at most
@@ -234,6 +238,12 @@ GAR_API int gar_plan_prepare(gar_plan *plan, int mode);
  * the last bits between ranks (each rank's association order is a rotation of the same
  * tree).  The modes give identical bits. */
 GAR_API int gar_allreduce(gar_plan *plan, void *const *rank_buffers, int mode, gar_stream_t stream);
+/* The plan is not const in gar_allreduce, gar_allreduce_host and gar_allreduce_batched:
+ * the first call on a device compiles and loads the plan's kernels, uploads its tables
+ * and records the stream and step counts it ran with -- state that gar_plan_status and
+ * gar_last_step_bytes read; the schedule itself never changes.
+ * In GAR_STEP_PERSISTENT mode the return value only says that the launch was enqueued:
+ * the results are complete only once gar_plan_status returns GAR_OK for the call. */
 
 /* Host-buffer Allreduce: the P inputs host_in[x] are in host memory and the P results
  * go to host memory host_out[x] (host_out[x] may equal host_in[x], or another rank's
@@ -273,18 +283,23 @@ GAR_API int gar_plan_status(gar_plan *plan);
 
 /* Barrier parameters of GAR_STEP_PERSISTENT (no counterpart in the paper).  spin_limit: polls (each an L2 round trip
  * plus a 64 ns sleep) a CTA makes at a grid barrier before it gives up (0 restores the
- * default, 2^20, roughly a second).
+ * default: 2^20 polls, roughly a second, or one poll per 256 bytes of memory traffic of
+ * the plan's largest step if that is more -- a wait then outlasts that step many times
+ * over).
  * phantom: extra arrivals the barrier waits for beyond the launched CTAs -- nonzero
  * values make every wait run out, which tests the timeout path without faulting
  * anything; keep 0 otherwise. */
 GAR_API int gar_plan_debug_barrier(gar_plan *plan, unsigned int phantom, unsigned int spin_limit);
 
 /* Bytes each communication step of the most recent step-faithful Allreduce read from
- * partner ranks, as counted by the kernels (S entries).  Synchronizes with the stream
- * of that call. */
+ * partner ranks, as counted by the kernels (S entries): the measured counterpart of the
+ * per-step message volume of gar_plan_bytes (Sec. "Communication operator"); the
+ * counting itself has no counterpart in the paper.  Synchronizes with the stream of
+ * that call; GAR_ESTATE if no step-faithful call ran. */
 GAR_API int gar_last_step_bytes(const gar_plan *plan, uint64_t *per_step);
 
-/* Name of a GAR_* status code (static string). */
+/* Name of a GAR_* status code (static string).  Error reporting; no counterpart in the
+ * paper. */
 GAR_API const char *gar_strerror(int status);
 /* The calling thread's most recent error detail (valid until its next failing call). */
 GAR_API const char *gar_last_error(void);
@@ -317,17 +332,22 @@ GAR_API int gar_optimal_steps(int P, double m_bytes, double alpha, double beta, 
  * run an Allreduce, e.g. code whose device memory is all owned by a caching
  * allocator or by another runtime.  Same result as gar_allreduce(plan, rank_buffers,
  * GAR_STEP_FAITHFUL, stream), but the workspace is a fixed file-scope device array of
- * GAR_NOALLOC_SCRATCH_BYTES, reserved on every GPU that loads the library until the
- * process exits, and the block ops travel in the kernel parameters; the plan's workspace
- * and device tables are not used, no bytes are recorded, and no cudaMalloc, cudaFree or
- * other allocating call is made.
+ * GAR_NOALLOC_SCRATCH_BYTES and the block ops travel in the kernel parameters; the
+ * plan's workspace and device tables are not used, no bytes are recorded, and no
+ * cudaMalloc, cudaFree or other allocating call is made.
+ * The array exists on a device once the library's step kernels are loaded there; CUDA
+ * loads them lazily: at the first step-faithful or persistent Allreduce, at
+ * gar_plan_prepare(plan, GAR_STEP_FAITHFUL or GAR_STEP_PERSISTENT), or at the first call
+ * of this function.  A caller whose allocator later takes all free memory should do one
+ * of these first; the array then stays until the process exits.
  * Limits: P <= GAR_NOALLOC_MAX_P and a workspace (gar_plan_bytes) of at most
  * GAR_NOALLOC_SCRATCH_BYTES; larger plans return GAR_EINVAL with the sizes in
- * gar_last_error().  The first call on a device looks up the array's device address
- * (cudaGetSymbolAddress) with that device current; make that first call before any
- * stream capture.  All calls share the one array and leave their partial results in it:
- * calls whose work overlaps on the GPU (other streams, other host threads) race, so
- * order them on one stream.  rank_buffers: as for gar_allreduce. */
+ * gar_last_error().  Every call looks up the array's address on the current device
+ * (cudaGetSymbolAddress, which allocates nothing); make the first call on a device, or
+ * the gar_plan_prepare above, before any stream capture.  All calls share the one array
+ * and leave their partial results in it: calls whose work overlaps on the GPU (other
+ * streams, other host threads) race, so order them on one stream.  rank_buffers: as for
+ * gar_allreduce. */
 #define GAR_NOALLOC_SCRATCH_BYTES (64u << 20)
 #define GAR_NOALLOC_MAX_P 64
 GAR_API int gar_allreduce_noalloc(gar_plan *plan, void *const *rank_buffers, gar_stream_t stream);

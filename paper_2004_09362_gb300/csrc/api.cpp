@@ -56,9 +56,22 @@ int ensure_device(gar_plan *pl) {
   return GAR_OK;
 }
 
+// Default poll limit of the persistent kernel's grid barriers: 2^20 polls (about a
+// second), or one poll per 256 bytes that the plan's largest step reads and writes (a
+// combine step: partner read, own read, write -- at most 3x its message bytes), so that
+// a legitimate wait never runs out however large the vectors are.
+unsigned int default_spin_limit(const gar_plan &pl) {
+  uint64_t most = 0;
+  for (const CommStep &cs : pl.comm) most = std::max<uint64_t>(most, 3 * cs.msg_bytes);
+  const uint64_t polls = std::max<uint64_t>(1u << 20, most / 256);
+  return (unsigned int)std::min<uint64_t>(polls, 0xffffffffull);
+}
+
 int prepare_step_faithful(gar_plan *pl) {
   int rc = ensure_device(pl);
   if (rc) return rc;
+  // the step kernels' module, loaded now rather than at the first launch
+  if ((rc = load_step_module())) return rc;
   if (pl->d_ops == nullptr && !pl->ops.empty()) {
     cudaError_t e = cudaMalloc(&pl->d_ops, pl->ops.size() * sizeof(StepOp));
     if (e != cudaSuccess) return cuda_fail(e, "cudaMalloc(op table)");
@@ -423,6 +436,7 @@ int gar_plan_create_group(gar_plan **out, int P, uint64_t n, int dtype, int op, 
     delete pl;
     return rc;
   }
+  pl->barrier_spin_limit = default_spin_limit(*pl);
   *out = pl;
   return GAR_OK;
 }
@@ -724,7 +738,7 @@ int gar_plan_status(gar_plan *pl) {
 int gar_plan_debug_barrier(gar_plan *pl, unsigned int phantom, unsigned int spin_limit) {
   if (int rc = check_plan(pl)) return rc;
   pl->barrier_phantom = phantom;
-  pl->barrier_spin_limit = spin_limit ? spin_limit : (1u << 20);
+  pl->barrier_spin_limit = spin_limit ? spin_limit : default_spin_limit(*pl);
   return GAR_OK;
 }
 

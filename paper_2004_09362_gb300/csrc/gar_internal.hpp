@@ -108,7 +108,7 @@ struct gar_plan {
   // persistent step-faithful mode: launch table, barrier state, barrier parameters
   void *d_launches = nullptr;
   void *d_barrier = nullptr;
-  unsigned int barrier_spin_limit = 1u << 20;   // polls: ~0.5-1 s (each is an L2 round trip + 64 ns)
+  unsigned int barrier_spin_limit = 1u << 20;   // polls (each an L2 round trip + 64 ns); see default_spin_limit
   unsigned int barrier_phantom = 0;
   bool ran_persistent = false;
   // pipelined host-buffer path: 3 streams (to device, kernel, to host) and events
@@ -166,6 +166,7 @@ int launch_step(const gar_plan &pl, const Launch &ln, int launch_index, void *co
                 gar_stream_t stream);
 int launch_persistent(const gar_plan &pl, void *const *rank, gar_stream_t stream);
 size_t barrier_state_bytes();
+int load_step_module();
 
 // api.cpp
 void set_error(const std::string &msg);

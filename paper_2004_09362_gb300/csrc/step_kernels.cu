@@ -17,7 +17,6 @@
 
 #include <algorithm>
 #include <cstdint>
-#include <mutex>
 #include <string>
 #include <type_traits>
 
@@ -266,20 +265,27 @@ __device__ __forceinline__ void chunk_work(const StepArgs<MAXP> &a, const Launch
   };
   const bool copy_only = kCopyPaths && !out1 && (has_recv != (own0 != nullptr));
   const uint8_t copy_src_buf = has_recv ? op.recv_buf : op.out0_own;
-  // A copy between buffers of one element type moves raw 4-element units (16 B, or 8 B
-  // for bf16) with a compile-time stride: few registers, so 6 units per thread in flight
-  // within the 40-register budget (8 spilled).
+  // A copy between buffers of one element type moves raw 16-byte units (4 fp32 or 8 bf16
+  // elements) with a compile-time stride: few registers, so 6 units per thread in flight
+  // within the 40-register budget.  bf16 copies used 8-byte units before and ran at
+  // about 4 TB/s (48 bytes in flight per thread) against 6.6 TB/s for fp32; elements
+  // before the first and after the last 16-byte boundary go one by one.
   auto raw_copy = [&](uint64_t va, uint64_t vb) {
-    using Vt = typename std::conditional<sizeof(T) == 2, uint2, int4>::type;
     constexpr int U = 6;
     const void *srcp = has_recv ? recv : own0;
     const uint64_t esz = copy_src_buf == BUF_RANK ? sizeof(T) : sizeof(A);
-    const Vt *src = reinterpret_cast<const Vt *>(static_cast<const char *>(srcp) + va * esz);
-    Vt *dst = reinterpret_cast<Vt *>(static_cast<char *>(out0) + va * esz);
-    const uint64_t units = (vb - va) / 4;
+    const uint64_t epu = 16 / esz;  // elements per 16-byte unit
+    uint64_t ua = (va + epu - 1) / epu * epu, ub = vb / epu * epu;
+    if (ua > vb) ua = vb;
+    if (ub < ua) ub = ua;
+    for (uint64_t e = va + threadIdx.x; e < ua; e += kThreads) do1(e);
+    for (uint64_t e = ub + threadIdx.x; e < vb; e += kThreads) do1(e);
+    const int4 *src = reinterpret_cast<const int4 *>(static_cast<const char *>(srcp) + ua * esz);
+    int4 *dst = reinterpret_cast<int4 *>(static_cast<char *>(out0) + ua * esz);
+    const uint64_t units = (ub - ua) / epu;
     for (uint64_t k = threadIdx.x; k < units; k += (uint64_t)U * kThreads) {
       const uint64_t left = units - k;
-      Vt v[U];
+      int4 v[U];
 #pragma unroll
       for (int u = 0; u < U; ++u)
         if ((uint64_t)u * kThreads < left) v[u] = src[k + (uint64_t)u * kThreads];
@@ -288,7 +294,7 @@ __device__ __forceinline__ void chunk_work(const StepArgs<MAXP> &a, const Launch
         if ((uint64_t)u * kThreads < left) dst[k + (uint64_t)u * kThreads] = v[u];
       if (has_recv) {
         const uint64_t cnt = left < (uint64_t)(U - 1) * kThreads + 1 ? (left + kThreads - 1) / kThreads : U;
-        moved += 4 * cnt;
+        moved += epu * cnt;
       }
     }
   };
@@ -582,18 +588,22 @@ __global__ void __launch_bounds__(kThreads) step_kernel_persistent(const __grid_
   }
 }
 
+// SM count of the current device (cached per device ordinal).
 int num_sms() {
-  static int sms = 0;
-  if (sms == 0) {
-    int dev = 0, v = 0;
-    cudaGetDevice(&dev);
-    if (cudaDeviceGetAttribute(&v, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess || v <= 0) {
-      cudaGetLastError();
-      v = 1;
-    }
-    sms = v;
+  static int cache[64] = {};
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0) {
+    cudaGetLastError();
+    dev = 0;
   }
-  return sms;
+  if (dev < 64 && cache[dev] > 0) return cache[dev];
+  int v = 0;
+  if (cudaDeviceGetAttribute(&v, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess || v <= 0) {
+    cudaGetLastError();
+    v = 1;
+  }
+  if (dev < 64) cache[dev] = v;
+  return v;
 }
 
 template <typename T, int OP, int MAXP>
@@ -631,9 +641,18 @@ int launch_typed(const gar_plan &pl, const Launch &ln, int launch_index, void *c
     if (e != cudaSuccess) return cuda_fail(e, "step kernel launch");
     return GAR_OK;
   }
-  a.chunk = kChunk;
+  // Distribution steps copy 2-byte elements with as many bytes per CTA as fp32 chunks
+  // hold; a last chunk shorter than 1/8 of a chunk is spread over the block's others (P =
+  // 127 x 8 MiB bf16: blocks of 33,026 elements became 16,384 + 16,384 + 258, a third of
+  // the CTAs nearly empty).
+  a.chunk = (ln.phase == 1 && sizeof(T) == 2) ? 2 * kChunk : kChunk;
   const uint64_t min_ctas = 4 * (uint64_t)num_sms();
   while (a.chunk > 4096 && ((maxblk + a.chunk - 1) / a.chunk) * pl.P * ln.nops < min_ctas) a.chunk /= 2;
+  {
+    const uint64_t nch = (maxblk + a.chunk - 1) / a.chunk;
+    if (nch > 1 && maxblk - (nch - 1) * a.chunk < a.chunk / 8)
+      a.chunk = ((maxblk + nch - 2) / (nch - 1) + 7) / 8 * 8;
+  }
   a.nchunks = (int)((maxblk + a.chunk - 1) / a.chunk);
   if (a.nchunks == 0 || ln.nops == 0) return GAR_OK;
   const uint64_t grid = (uint64_t)a.nchunks * (uint64_t)pl.P * (uint64_t)ln.nops;
@@ -749,8 +768,10 @@ size_t barrier_state_bytes() { return sizeof(BarrierState); }
 // no allocator hook -- the workspace lives in one file-scope device array of fixed
 // size instead of a caller-supplied buffer, and each launch receives its block ops by
 // value in the kernel parameters instead of from a device table.  No cudaMalloc,
-// cudaFree or memset is issued.  The array is reserved on every device that loads
-// this library and stays reserved until the process exits.  Nothing in it needs to
+// cudaFree or memset is issued.  The array exists on a device once this file's device
+// code is loaded there -- under CUDA's lazy module loading, at the first launch of any
+// of its kernels, at gar_plan_prepare of a step-faithful mode, or at the first
+// no-allocation call -- and stays until the process exits.  Nothing in it needs to
 // start at zero: the schedule writes every workspace slot before it reads it.  All
 // calls share the array, so two calls whose work overlaps on the GPU race.
 // ---------------------------------------------------------------------------
@@ -846,27 +867,26 @@ __global__ void __launch_bounds__(kThreads) step_kernel_noalloc(const __grid_con
   for (uint64_t e = vb + threadIdx.x; e < hi; e += blockDim.x) do1(e);
 }
 
-std::mutex g_noalloc_mu;
-void *g_noalloc_ptr[64] = {};
+// Device address of the scratch array on the current device, looked up on every call
+// with that device current: the lookup allocates nothing, and a cached address would be
+// stale after cudaDeviceReset or in another context on the same device.
+int noalloc_scratch(void **out);
 
-// Device address of the scratch array on the current device.  The first call on a
-// device resolves it (with that device current) and caches it; later calls reuse it.
+}  // namespace
+
+// Loads this file's device code on the current device (and with it the scratch array).
+int load_step_module() {
+  void *p = nullptr;
+  return noalloc_scratch(&p);
+}
+
+namespace {
+
 int noalloc_scratch(void **out) {
-  int dev = -1;
-  cudaError_t e = cudaGetDevice(&dev);
-  if (e != cudaSuccess) return cuda_fail(e, "cudaGetDevice");
-  if (dev < 0 || dev >= 64) {
-    set_error("device ordinal out of range for the no-allocation scratch table");
-    return GAR_EINVAL;
-  }
-  std::lock_guard<std::mutex> lock(g_noalloc_mu);
-  if (g_noalloc_ptr[dev] == nullptr) {
-    void *p = nullptr;
-    e = cudaGetSymbolAddress(&p, g_noalloc_scratch);
-    if (e != cudaSuccess) return cuda_fail(e, "cudaGetSymbolAddress(no-allocation scratch)");
-    g_noalloc_ptr[dev] = p;
-  }
-  *out = g_noalloc_ptr[dev];
+  void *p = nullptr;
+  cudaError_t e = cudaGetSymbolAddress(&p, g_noalloc_scratch);
+  if (e != cudaSuccess) return cuda_fail(e, "cudaGetSymbolAddress(no-allocation scratch)");
+  *out = p;
   return GAR_OK;
 }
 
