@@ -185,11 +185,11 @@ class L2Flusher:
 
     def __init__(self, nbytes=512 << 20):
         import torch
-        self.buf = torch.zeros(nbytes // 4, dtype=torch.int32, device="cuda")
-        self.acc = torch.int64
+        # float32 reduces in place of its own type: no widening copy (which would write)
+        self.buf = torch.zeros(nbytes // 4, dtype=torch.float32, device="cuda")
 
     def __call__(self):
-        self.buf.sum(dtype=self.acc)
+        self.buf.sum()
 
 
 # ---------------------------------------------------------------------------
@@ -653,7 +653,7 @@ def cost_model_row(gar, gar_inputs, stream, hbm_peak, P=127, dtype="bf16",
     from scipy.optimize import nnls
     es = 2 if dtype == "bf16" else 4
     L = _l(P)
-    times = {}
+    times, dram = {}, {}
     for m in sizes:
         n = max(1, m // es)
         raw = gar_inputs.rank_inputs(P, n, dtype, ("normal", 0.0, 1.0), 77, device="cuda")
@@ -668,6 +668,7 @@ def cost_model_row(gar, gar_inputs, stream, hbm_peak, P=127, dtype="bf16",
             reps = 20 if m <= (64 << 10) else 5
             times[(m, S)] = _time_loop(lambda: gar.gar_allreduce(plan, inp, "step", stream), reps, 3,
                                        stream) * 1e-3
+            dram[(m, S)] = _step_dram_bytes(gar, plan, P, n, dtype)
             plan.workspace = None
             del plan
             torch.cuda.empty_cache()
@@ -713,8 +714,21 @@ def cost_model_row(gar, gar_inputs, stream, hbm_peak, P=127, dtype="bf16",
                 for m in sizes}
     per_step_us = {str(m): {f"S{S}": round(times[(m, S)] * 1e6 / S, 2) for S in range(L, 2 * L + 1)}
                    for m in sizes}
+    # Where the paper's linear per-message model breaks on this machine: a step that moves
+    # d DRAM bytes should take alpha + d / HBM; the effective DRAM rate of each schedule
+    # shows how far below HBM the small-message steps run (per-item latency, not bytes).
+    eff = {str(m): {f"S{S}": round(dram[(m, S)] / times[(m, S)] / 1e9, 1) for S in range(L, 2 * L + 1)}
+           for m in sizes}
+    m_lo, m_hi = sizes[1], sizes[-1]
+    violation = (
+        f"beta is not constant: the step-faithful Allreduce moves its DRAM-model bytes at "
+        f"{eff[str(m_hi)][f'S{2 * L}']} GB/s (S={2 * L}) and {eff[str(m_hi)][f'S{L}']} GB/s (S={L}) "
+        f"at {m_hi} B per rank, but at {eff[str(m_lo)][f'S{2 * L}']} and {eff[str(m_lo)][f'S{L}']} GB/s "
+        f"at {m_lo} B: below a few MB per step a launch is too small to reach HBM bandwidth, so the "
+        f"cost of a byte grows as the blocks shrink, most for the many-block steps of small S")
     return {"P": P, "dtype": dtype, "mode": "step", "measured_us": measured,
-            "measured_us_per_step": per_step_us,
+            "measured_us_per_step": per_step_us, "effective_dram_GBps": eff,
+            "linear_model_violation": violation,
             "fit_free": evaluate(*fitted), "fit_derived": evaluate(*derived),
             "derived_from": f"alpha: slope of time over S at {sizes[0]} B; beta = P / HBM, "
                             f"gamma = 2P / HBM with HBM = {hbm_peak} GB/s (measured copy)"}
