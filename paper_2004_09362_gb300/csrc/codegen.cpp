@@ -59,6 +59,25 @@ static __device__ __forceinline__ gar_acc gar_op(gar_acc a, gar_acc b) {
 #endif
 }
 
+// out[w] = a[w] (+) b[w] for W element positions; float sums of an even W pair the
+// positions in paired fp32 adds (__fadd2_rn: round to nearest even in each half)
+template <int W>
+static __device__ __forceinline__ void gar_comb(gar_acc *out, const gar_acc *a, const gar_acc *b) {
+#if GAR_DTYPE != 2 && GAR_OP == 0 && GAR_FADD2
+  if (W % 2 == 0) {
+#pragma unroll
+    for (int w = 0; w < W; w += 2) {
+      const float2 r = __fadd2_rn(make_float2(a[w], a[w + 1]), make_float2(b[w], b[w + 1]));
+      out[w] = r.x;
+      out[w + 1] = r.y;
+    }
+    return;
+  }
+#endif
+#pragma unroll
+  for (int w = 0; w < W; ++w) out[w] = gar_op(a[w], b[w]);
+}
+
 static __device__ __forceinline__ float gar_bf16_lo(gar_u32 u) { return __uint_as_float(u << 16); }
 static __device__ __forceinline__ float gar_bf16_hi(gar_u32 u) { return __uint_as_float(u & 0xffff0000u); }
 static __device__ __forceinline__ gar_u32 gar_pack_bf16(float lo, float hi) {
@@ -281,7 +300,7 @@ std::string emit_eval(const FusedProgram &fp, const Schedule &sc, const std::str
            std::to_string(v) + ");\n";
     } else if (kind == 1) {
       const int a = fp.a[v - P], b = fp.b[v - P];
-      s += fmt("  gar_acc v%d[W];\n#pragma unroll\n  for (int w = 0; w < W; ++w) v%d[w] = gar_op(v%d[w], v%d[w]);\n",
+      s += fmt("  gar_acc v%d[W]; gar_comb<W>(v%d, v%d, v%d);\n",
                v, v, a, b);
     } else {
       const int val = fp.out[v];
@@ -341,6 +360,10 @@ CodegenResult generate_fused_source(const gar_plan &pl) {
                    op_tag(pl.op) + fmt("_W%d", W) + (pl.group == GAR_GROUP_XOR ? "_xor" : "");
   std::string s;
   s += fmt("#define GAR_DTYPE %d\n#define GAR_OP %d\n", pl.dtype, pl.op);
+  // paired fp32 adds over element positions for bf16 programs at W >= 4 (P = 127:
+  // S = 10 0.377 -> 0.360 ms, S = 11 0.354 -> 0.344 ms); fp32 programs and W = 2 were
+  // slower or spilled (P = 64 fp32, S = 8: 104 -> 255 registers)
+  s += fmt("#define GAR_FADD2 %d\n", tune_int("GAR_TUNE_FADD2", pl.dtype == GAR_BF16 && W >= 4) != 0 ? 1 : 0);
   s += "#define GAR_LDH \"" + tune_str("GAR_TUNE_LDH", ".cs") + "\"\n";
   s += "#define GAR_STH \"" + tune_str("GAR_TUNE_STH", ".cs") + "\"\n";
   s += kSkeleton;
@@ -666,6 +689,7 @@ CodegenResult generate_batched_source(const std::vector<const gar_plan *> &plans
   cg.kernel_name = name + dtype_tag(p0.dtype) + "_" + op_tag(p0.op) + fmt("_W%d", W);
   std::string s;
   s += fmt("#define GAR_DTYPE %d\n#define GAR_OP %d\n", p0.dtype, p0.op);
+  s += fmt("#define GAR_FADD2 %d\n", tune_int("GAR_TUNE_FADD2", 0) != 0 ? 1 : 0);
   s += "#define GAR_LDH \"" + tune_str("GAR_TUNE_LDH", ".cs") + "\"\n";
   s += "#define GAR_STH \"" + tune_str("GAR_TUNE_STH", ".cs") + "\"\n";
   s += kSkeleton;

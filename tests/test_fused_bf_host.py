@@ -57,8 +57,9 @@ def test_every_combine_emitted_once():
     """P = 127, S = 7: the 1524 combines are 2 x (paired adds) + single adds, and the
     even-distance steps pair most of them."""
     src, info = _bf_source(127, 4194304, "bf16", 7)
-    pairs = src.count("__fadd2_rn(make_float2(")
-    singles = len(re.findall(r"const gar_acc v\d+ = gar_(?:addbf|op)\(", src))
+    body = re.search(r"void gar_eval_bf\(.*?\n\}\n", src, re.S).group(0)
+    pairs = body.count("__fadd2_rn(make_float2(")
+    singles = len(re.findall(r"const gar_acc v\d+ = gar_(?:addbf|op)\(", body))
     assert 2 * pairs + singles == info["fused_combines"] == 1524
     assert pairs >= 500
     assert "__launch_bounds__(32, 8)" in src      # 254 live values: 255 registers
