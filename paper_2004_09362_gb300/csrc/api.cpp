@@ -144,6 +144,25 @@ int compile_fused(gar_plan *pl) {
   JitKernel *k = nullptr;
   int rc = jit_compile(cg, &k);
   if (rc) return rc;
+  // Register-heavy single-thread kernels (ptxas above 128 registers) run in 64-thread
+  // CTAs capped at 168 registers, so that three warps share each sub-partition's register
+  // file and the small CTAs of an SM drift apart.  On GB300: P = 32 x 32 MiB bf16
+  // latency-optimal (208 registers) 0.426 -> 0.338 ms; P = 127 x 8 MiB bf16 S = 9 (200)
+  // 0.434 -> 0.401 ms, S = 11 (174) 0.344 -> 0.324 ms; kernels at 128 registers or fewer
+  // were unchanged or slower (P = 64 fp32 latency-optimal, 40 registers: 0.33 -> 0.40 ms).
+  const bool shape_forced = std::getenv("GAR_TUNE_FUSED_THREADS") || std::getenv("GAR_TUNE_FUSED_MINB");
+  if (cg.form == 0 && !shape_forced && k->ptxas_regs > 128) {
+    CodegenResult cg2;
+    try {
+      cg2 = generate_fused_source(*pl, 64, 5);
+    } catch (const std::exception &ex) {
+      set_error(std::string("fused code generation: ") + ex.what());
+      return GAR_EINVAL;
+    }
+    JitKernel *k2 = nullptr;
+    if ((rc = jit_compile(cg2, &k2))) return rc;
+    k = k2;
+  }
   pl->fused = k;
   pl->fused_width = k->width;
   return GAR_OK;
@@ -558,7 +577,7 @@ int gar_plan_fused_source(const gar_plan *pl, char *buf, size_t *len) {
   if (len == nullptr) return GAR_EINVAL;
   std::string src;
   try {
-    src = fused_codegen(*pl).source;
+    src = pl->fused != nullptr ? pl->fused->source : fused_codegen(*pl).source;
   } catch (const std::exception &ex) {
     set_error(std::string("fused code generation: ") + ex.what());
     return GAR_EINVAL;

@@ -333,7 +333,7 @@ std::string emit_block_of(const std::string &name, int P, uint64_t n) {
 
 }  // namespace
 
-CodegenResult generate_fused_source(const gar_plan &pl) {
+CodegenResult generate_fused_source(const gar_plan &pl, int threads_override, int minb_override) {
   const FusedProgram &fp = pl.prog;
   const int P = pl.P;
   Schedule sc = order_program(fp);
@@ -348,8 +348,8 @@ CodegenResult generate_fused_source(const gar_plan &pl) {
   while (W > 1 && pl.n / (uint64_t)W < 16384) W /= 2;
   if (int w = tune_int("GAR_TUNE_FUSED_W", 0))
     if (w > 0 && (w & (w - 1)) == 0 && w * elem_size(pl.dtype) <= 16) W = w;
-  const int minb = tune_int("GAR_TUNE_FUSED_MINB", 0);
-  int nthr = tune_int("GAR_TUNE_FUSED_THREADS", 256);
+  const int minb = minb_override > 0 ? minb_override : tune_int("GAR_TUNE_FUSED_MINB", 0);
+  int nthr = threads_override > 0 ? threads_override : tune_int("GAR_TUNE_FUSED_THREADS", 256);
   if (nthr < 32 || nthr > 1024 || nthr % 32 != 0) nthr = 256;
   const std::string bounds = minb > 0 ? fmt("__launch_bounds__(%d, %d)", nthr, minb)
                                       : fmt("__launch_bounds__(%d)", nthr);

@@ -137,7 +137,8 @@ struct CodegenResult {
   int threads = 256;     // threads per CTA
   int form = 0;          // fused kernels: 0 single-thread program, 1 breadth-first
 };
-CodegenResult generate_fused_source(const gar_plan &pl);
+// threads / minb > 0 override the CTA size and the minimum resident CTAs per SM
+CodegenResult generate_fused_source(const gar_plan &pl, int threads = 0, int minb = 0);
 // The breadth-first form of the fused kernel (programs with many result copies), and
 // the peak number of live values of a plan's program in the single-thread form.
 CodegenResult generate_fused_bf_source(const gar_plan &pl);
@@ -149,6 +150,7 @@ struct JitKernel {
   void *library = nullptr;   // cudaLibrary_t
   void *kernel = nullptr;    // cudaKernel_t
   std::vector<char> cubin;
+  std::string source;        // the generated CUDA source it was compiled from
   std::string name;
   int width = 1;
   int table_copies = 1;
@@ -156,6 +158,7 @@ struct JitKernel {
   int form = 0;
   int blocks_per_sm = 0;
   int regs = 0, local_bytes = 0;
+  int ptxas_regs = 0;        // registers per thread as ptxas reported them at compile time
   bool loaded = false;
 };
 int jit_compile(const CodegenResult &cg, JitKernel **out);
