@@ -503,6 +503,7 @@ def measure_rows(gar, gar_inputs, stream, hbm_peak):
                "fused_frac": round(_alg_bytes(P, n, "bf16") / ms_f / 1e6 / hbm_peak, 4),
                "fused_combines_per_position": plan.info()["fused_combines"],
                "fused_width": plan.info()["fused_width"],
+               "fused_regs": plan.info()["fused_regs"],
                "fused_form": "breadth_first" if plan.info()["fused_form"] == 1 else "single"}
         if S in (7, 10, 14):
             gar.ensure_workspace(plan)

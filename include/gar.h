@@ -216,9 +216,9 @@ GAR_API int gar_plan_step_ops(const gar_plan *plan, int32_t *ops, int *nops, int
 GAR_API int gar_plan_set_workspace(gar_plan *plan, void *dev_ptr, size_t bytes);
 
 /* The CUDA C source of the plan's generated fused kernel (host-only): of the kernel the
- * plan runs once it is compiled (gar_plan_compile, gar_plan_prepare or a first fused
- * call: register-heavy kernels are then recompiled in smaller CTAs), else of the first
- * compile.  Copies at most
+ * plan runs once it is prepared (gar_plan_prepare or a first fused call, which rebuild a
+ * kernel of more than 128 registers in 64-thread CTAs), else of its first compile.
+ * Copies at most
  * *len bytes (including the terminating NUL) to buf and sets *len to the full size
  * including the NUL; pass buf == NULL to query the size. */
 GAR_API int gar_plan_fused_source(const gar_plan *plan, char *buf, size_t *len);

@@ -144,36 +144,40 @@ int compile_fused(gar_plan *pl) {
   JitKernel *k = nullptr;
   int rc = jit_compile(cg, &k);
   if (rc) return rc;
-  // Register-heavy single-thread kernels (ptxas above 128 registers) run in 64-thread
-  // CTAs capped at 168 registers, so that three warps share each sub-partition's register
-  // file and the small CTAs of an SM drift apart.  On GB300: P = 32 x 32 MiB bf16
-  // latency-optimal (208 registers) 0.426 -> 0.338 ms; P = 127 x 8 MiB bf16 S = 9 (200)
-  // 0.434 -> 0.401 ms, S = 11 (174) 0.344 -> 0.324 ms; kernels at 128 registers or fewer
-  // were unchanged or slower (P = 64 fp32 latency-optimal, 40 registers: 0.33 -> 0.40 ms).
-  const bool shape_forced = std::getenv("GAR_TUNE_FUSED_THREADS") || std::getenv("GAR_TUNE_FUSED_MINB");
-  if (cg.form == 0 && !shape_forced && k->ptxas_regs > 128) {
-    CodegenResult cg2;
-    try {
-      cg2 = generate_fused_source(*pl, 64, 5);
-    } catch (const std::exception &ex) {
-      set_error(std::string("fused code generation: ") + ex.what());
-      return GAR_EINVAL;
-    }
-    JitKernel *k2 = nullptr;
-    if ((rc = jit_compile(cg2, &k2))) return rc;
-    k = k2;
-  }
   pl->fused = k;
   pl->fused_width = k->width;
   return GAR_OK;
 }
 
+// Register-heavy single-thread kernels (more than 128 registers once loaded) run in
+// 64-thread CTAs capped at 168 registers, so that three warps share each sub-partition's
+// register file and the small CTAs of an SM drift apart.  On GB300: P = 32 x 32 MiB bf16
+// latency-optimal (208 registers) 0.426 -> 0.338 ms; P = 127 x 8 MiB bf16 S = 9 (200)
+// 0.434 -> 0.401 ms, S = 11 (174) 0.344 -> 0.324 ms; kernels at 128 registers or fewer
+// were unchanged or slower (P = 64 fp32 latency-optimal, 40 registers: 0.33 -> 0.40 ms).
+// The count is the loaded kernel's own (the compiler's log does not always carry it).
 int prepare_fused(gar_plan *pl) {
   int rc = compile_fused(pl);
   if (rc) return rc;
   rc = ensure_device(pl);
   if (rc) return rc;
-  return jit_load(pl->fused);
+  if ((rc = jit_load(pl->fused))) return rc;
+  const bool shape_forced = std::getenv("GAR_TUNE_FUSED_THREADS") || std::getenv("GAR_TUNE_FUSED_MINB");
+  if (pl->fused->form == 0 && pl->fused->threads == 256 && !shape_forced && pl->fused->regs > 128) {
+    CodegenResult cg;
+    try {
+      cg = generate_fused_source(*pl, 64, 5);
+    } catch (const std::exception &ex) {
+      set_error(std::string("fused code generation: ") + ex.what());
+      return GAR_EINVAL;
+    }
+    JitKernel *k = nullptr;
+    if ((rc = jit_compile(cg, &k))) return rc;
+    if ((rc = jit_load(k))) return rc;
+    pl->fused = k;
+    pl->fused_width = k->width;
+  }
+  return GAR_OK;
 }
 
 int check_buffers(const gar_plan *pl, void *const *bufs) {

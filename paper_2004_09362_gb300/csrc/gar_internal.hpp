@@ -158,7 +158,6 @@ struct JitKernel {
   int form = 0;
   int blocks_per_sm = 0;
   int regs = 0, local_bytes = 0;
-  int ptxas_regs = 0;        // registers per thread as ptxas reported them at compile time
   bool loaded = false;
 };
 int jit_compile(const CodegenResult &cg, JitKernel **out);

@@ -6,7 +6,6 @@
 #include <cuda_runtime.h>
 #include <nvrtc.h>
 
-#include <cstdlib>
 #include <memory>
 #include <mutex>
 #include <string>
@@ -35,11 +34,8 @@ int jit_compile(const CodegenResult &cg, JitKernel **out) {
     set_error("nvrtcCreateProgram failed");
     return GAR_EJIT;
   }
-  // ptxas reports its register count in the log (-v); the fused kernels' launch shape
-  // depends on it (compile_fused)
   const char *opts[] = {"--gpu-architecture=sm_103a", "--std=c++17", "-lineinfo",
-                        "--fmad=false", "--ftz=false", "--prec-div=true", "--prec-sqrt=true",
-                        "--ptxas-options=-v"};
+                        "--fmad=false", "--ftz=false", "--prec-div=true", "--prec-sqrt=true"};
   nvrtcResult rc = nvrtcCompileProgram(prog, (int)(sizeof opts / sizeof opts[0]), opts);
   if (rc != NVRTC_SUCCESS) {
     size_t n = 0;
@@ -57,14 +53,6 @@ int jit_compile(const CodegenResult &cg, JitKernel **out) {
     return GAR_EJIT;
   }
   auto k = std::make_unique<JitKernel>();
-  {
-    size_t n = 0;
-    nvrtcGetProgramLogSize(prog, &n);
-    std::string log(n, '\0');
-    if (n) nvrtcGetProgramLog(prog, &log[0]);
-    const size_t at = log.find("Used ");
-    if (at != std::string::npos) k->ptxas_regs = std::atoi(log.c_str() + at + 5);
-  }
   k->cubin.resize(bytes);
   nvrtcGetCUBIN(prog, k->cubin.data());
   nvrtcDestroyProgram(&prog);

@@ -211,14 +211,3 @@ def test_breadth_first_kernels_compile(P):
             G.gar_plan_compile(G.gar_plan_create_group(P, 1000, "f32", "sum", L, "xor"), "fused")
     _with_form(1, go)
 
-
-def test_register_heavy_single_kernels_get_small_ctas():
-    """After compiling, a single-thread kernel that ptxas builds with more than 128
-    registers is rebuilt in 64-thread CTAs capped at 168 registers; lighter ones keep
-    256-thread CTAs."""
-    heavy = G.gar_plan_create(127, 4194304, "bf16", "sum", 9)
-    G.gar_plan_compile(heavy, "fused")
-    assert "__launch_bounds__(64, 5)" in G.gar_plan_fused_source(heavy)
-    light = G.gar_plan_create(24, 1 << 24, "f32", "sum", 10)
-    G.gar_plan_compile(light, "fused")
-    assert "__launch_bounds__(256)" in G.gar_plan_fused_source(light)

@@ -262,6 +262,18 @@ def test_breadth_first_form_every_step_count(P, n, dtype, op, monkeypatch):
         _assert_same(_run(plan, t, "fused"), G.allreduce(host, S, op, dtype), dtype, f"S={S}")
 
 
+def test_register_heavy_single_kernels_get_small_ctas():
+    """Once prepared, a single-thread kernel of more than 128 registers runs in 64-thread
+    CTAs capped at 168 registers; lighter ones keep 256-thread CTAs."""
+    heavy = gar.gar_plan_create(127, 4194304, "bf16", "sum", 9)
+    gar.gar_plan_prepare(heavy, "fused")
+    assert "__launch_bounds__(64, 5)" in gar.gar_plan_fused_source(heavy)
+    assert gar.gar_plan_get_info(heavy)["fused_regs"] <= 168
+    light = gar.gar_plan_create(24, 1 << 24, "f32", "sum", 10)
+    gar.gar_plan_prepare(light, "fused")
+    assert "__launch_bounds__(256)" in gar.gar_plan_fused_source(light)
+
+
 @pytest.mark.parametrize("P", [8, 32])
 def test_breadth_first_form_xor_group(P, monkeypatch):
     monkeypatch.setenv("GAR_TUNE_FUSED_FORM", "1")
