@@ -123,11 +123,16 @@ int check_fused_size(const gar_plan *pl) {
 // breadth-first form (0.59 instead of 0.68 ms, and 0.47 instead of 0.56 ms, at P = 127 x
 // 8 MiB bf16 on GB300); every other plan takes the single-thread form.  GAR_TUNE_FUSED_FORM
 // (0 or 1) forces one form, for parity tests and launch-shape sweeps.
-CodegenResult fused_codegen(const gar_plan &pl) {
+int fused_form(const gar_plan &pl) {
+  if (pl.K <= 1) return GAR_FORM_SINGLE;
   const char *ff = std::getenv("GAR_TUNE_FUSED_FORM");
-  int form = (pl.K > 1 && pl.op == GAR_SUM && pl.dtype != GAR_I32 && fused_peak_live(pl) > 160) ? 1 : 0;
-  if (ff && *ff) form = std::atoi(ff) == 1 ? 1 : 0;
-  if (form == 1 && pl.K > 1) return generate_fused_bf_source(pl);
+  if (ff && *ff) return std::atoi(ff) == 1 ? GAR_FORM_BREADTH : GAR_FORM_SINGLE;
+  return (pl.op == GAR_SUM && pl.dtype != GAR_I32 && fused_peak_live(pl) > 160) ? GAR_FORM_BREADTH
+                                                                                : GAR_FORM_SINGLE;
+}
+
+CodegenResult fused_codegen(const gar_plan &pl) {
+  if (fused_form(pl) == GAR_FORM_BREADTH) return generate_fused_bf_source(pl);
   return generate_fused_source(pl);
 }
 
@@ -498,7 +503,7 @@ int gar_plan_get_info(const gar_plan *pl, gar_plan_info *info) {
   info->fused_combines = (int)pl->prog.a.size();
   info->group = pl->group;
   info->ring = pl->ring ? 1 : 0;
-  info->fused_form = pl->K > 1 ? fused_codegen(*pl).form : GAR_FORM_SINGLE;
+  info->fused_form = pl->fused != nullptr ? pl->fused->form : fused_form(*pl);
   info->fused_width = pl->fused_width;
   if (pl->fused != nullptr && pl->fused->loaded) {
     info->fused_regs = pl->fused->regs;
