@@ -160,7 +160,14 @@ int compile_fused(gar_plan *pl) {
 // latency-optimal (208 registers) 0.426 -> 0.338 ms; P = 127 x 8 MiB bf16 S = 9 (200)
 // 0.434 -> 0.401 ms, S = 11 (174) 0.344 -> 0.324 ms; kernels at 128 registers or fewer
 // were unchanged or slower (P = 64 fp32 latency-optimal, 40 registers: 0.33 -> 0.40 ms).
-// The count is the loaded kernel's own (the compiler's log does not always carry it).
+// When the 168-register build spills more than 256 bytes per thread, 32-thread CTAs with
+// the full 255 registers (two warps per sub-partition) are built too and kept if they
+// spill less: P = 127 x 8 MiB bf16 S = 10 (168 registers + 328 B spilled, 0.369 ms;
+// 250 registers, no spill, 0.351 ms).  Smaller spills cost less than the lost warps:
+// P = 32 x 32 MiB bf16 S = 5 (152 B: 0.341 ms against 0.390 ms at 210 registers),
+// P = 64 x 16 MiB bf16 S = 8 (96 B: 0.324 against 0.346), P = 127 S = 9 (48 B: 0.407
+// against 0.460).
+// The counts are the loaded kernel's own (the compiler's log does not always carry them).
 int prepare_fused(gar_plan *pl) {
   int rc = compile_fused(pl);
   if (rc) return rc;
@@ -168,20 +175,28 @@ int prepare_fused(gar_plan *pl) {
   if (rc) return rc;
   if ((rc = jit_load(pl->fused))) return rc;
   const bool shape_forced = std::getenv("GAR_TUNE_FUSED_THREADS") || std::getenv("GAR_TUNE_FUSED_MINB");
-  if (pl->fused->form == 0 && pl->fused->threads == 256 && !shape_forced && pl->fused->regs > 128) {
+  if (pl->fused->form != 0 || pl->fused->threads != 256 || shape_forced || pl->fused->regs <= 128)
+    return GAR_OK;
+  auto build = [&](int threads, int minb, JitKernel **out) -> int {
     CodegenResult cg;
     try {
-      cg = generate_fused_source(*pl, 64, 5);
+      cg = generate_fused_source(*pl, threads, minb);
     } catch (const std::exception &ex) {
       set_error(std::string("fused code generation: ") + ex.what());
       return GAR_EINVAL;
     }
-    JitKernel *k = nullptr;
-    if ((rc = jit_compile(cg, &k))) return rc;
-    if ((rc = jit_load(k))) return rc;
-    pl->fused = k;
-    pl->fused_width = k->width;
+    if (int r = jit_compile(cg, out)) return r;
+    return jit_load(*out);
+  };
+  JitKernel *k = nullptr;
+  if ((rc = build(64, 5, &k))) return rc;
+  if (k->local_bytes > 256) {
+    JitKernel *wide = nullptr;
+    if ((rc = build(32, 8, &wide))) return rc;
+    if (wide->local_bytes < k->local_bytes) k = wide;
   }
+  pl->fused = k;
+  pl->fused_width = k->width;
   return GAR_OK;
 }
 

@@ -169,7 +169,8 @@ template <> __device__ __forceinline__ void gar_store<4>(gar_io *p, const gar_ac
 // are part of the generated source, so kernels of different settings never share a cache
 // entry.  GAR_TUNE_FUSED_W: elements per thread-vector; GAR_TUNE_FUSED_MINB: minimum
 // resident CTAs per SM in __launch_bounds__; GAR_TUNE_LDH / GAR_TUNE_STH: cache-hint
-// suffix of the global loads / stores (default ".cs", streaming).
+// suffix of the global loads / stores (default ".cs", streaming); GAR_TUNE_DOUBLED (0 or
+// 1): whether a rotated cyclic single-thread kernel stores its pointer tables twice.
 int tune_int(const char *name, int dflt) {
   const char *v = std::getenv(name);
   return (v && *v) ? std::atoi(v) : dflt;
@@ -338,7 +339,9 @@ CodegenResult generate_fused_source(const gar_plan &pl, int threads_override, in
   const int P = pl.P;
   Schedule sc = order_program(fp);
   const bool rotate = pl.K != P;   // latency-optimal results do not depend on the block
-  const bool doubled = rotate && pl.group != GAR_GROUP_XOR && P <= 1000 && pl.K > 1;
+  bool doubled = rotate && pl.group != GAR_GROUP_XOR && P <= 1000 && pl.K > 1;
+  if (const int d = tune_int("GAR_TUNE_DOUBLED", -1); d >= 0)
+    doubled = d != 0 && rotate && pl.group != GAR_GROUP_XOR && P <= 1000;
   // bf16 programs with doubled pointer tables (below) run best with at most 8-byte
   // vectors (P = 127, S = 8..13: W = 8 was 3-6 % slower at S = 12, 13 than W = 4).
   int W = choose_width(pl.dtype, sc.peak_live, (doubled && pl.dtype == GAR_BF16) ? 4 : 16);
@@ -376,8 +379,10 @@ CodegenResult generate_fused_source(const gar_plan &pl, int threads_override, in
   // table twice turns that into b + j, which folds into the constant-bank offset of the
   // pointer load (the parameter block stays within 32 KB up to P = 1000).  Only for
   // programs with several result copies (K > 1): there it freed registers and made P = 127
-  // bf16 up to 19 % faster (S = 8..13); the single-copy programs (bandwidth-optimal, folds,
-  // the Ring) are HBM-bound and ran 0.6-0.8 % slower with it.
+  // bf16 up to 19 % faster (S = 8..13).  The single-copy programs (bandwidth-optimal, folds,
+  // the Ring) are HBM-bound and mostly ran slower with it: P = 24 x 64 MiB fp32 S = 10 by
+  // 0.8 %, P = 24 x 64 MiB bf16 S = 10 by 1.1 %, P = 8 x 256 MiB bf16 S = 6 by 4 %
+  // (P = 127 x 8 MiB bf16 S = 14 ran 1 % faster).
   cg.table_copies = doubled ? 2 : 1;
   s += fmt("struct gar_args { const gar_io *in[%d]; gar_io *out[%d]; gar_u64 e_lo, e_hi; };\n",
            cg.table_copies * P, cg.table_copies * P);
@@ -580,11 +585,12 @@ CodegenResult generate_fused_bf_source(const gar_plan &pl) {
   // Launch shape, from P = 127 x 8 MiB bf16 on GB300: the widest programs (S = 7, 254
   // live values) at 255 registers in 32-thread CTAs, 8 per SM (0.60 ms; 0.63 ms in
   // 64-thread CTAs); the others at 168 registers (a third warp per sub-partition register
-  // file) in 64-thread CTAs (S = 8, 192 live values: 0.47 ms; 0.60 ms at 255 registers).
+  // file) in 128-thread CTAs, 3 per SM (S = 8, 192 live values: 0.464 ms; 0.473 ms in
+  // 64-thread CTAs, 0.48 ms in 32-thread ones, 0.56-0.60 ms at 255 or 128 registers).
   const int peak = order_program(fp).peak_live;
   const bool widest = peak >= 224;
-  const int warps = std::max(1, std::min(16, tune_int("GAR_TUNE_BF_WARPS", widest ? 1 : 2)));
-  const int minb = std::max(1, tune_int("GAR_TUNE_BF_MINB", widest ? 8 : 5));
+  const int warps = std::max(1, std::min(16, tune_int("GAR_TUNE_BF_WARPS", widest ? 1 : 4)));
+  const int minb = std::max(1, tune_int("GAR_TUNE_BF_MINB", widest ? 8 : 3));
   // Pointer tables: the kernel parameters, indexed b + j (stored twice), while a warp's
   // 32 element positions share one block almost always (blocks of 32+ elements); with
   // shorter blocks the index differs across the lanes and the tables go to shared memory.

@@ -64,7 +64,7 @@ def test_every_combine_emitted_once():
     assert pairs >= 500
     assert "__launch_bounds__(32, 8)" in src      # 254 live values: 255 registers
     src8, _ = _bf_source(127, 4194304, "bf16", 8)
-    assert "__launch_bounds__(64, 5)" in src8     # 192 live values: 168 registers
+    assert "__launch_bounds__(128, 3)" in src8    # 192 live values: 168 registers
 
 
 # ---------------------------------------------------------------------------
