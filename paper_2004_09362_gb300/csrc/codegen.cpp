@@ -339,7 +339,18 @@ CodegenResult generate_fused_source(const gar_plan &pl, int threads_override, in
   const int P = pl.P;
   Schedule sc = order_program(fp);
   const bool rotate = pl.K != P;   // latency-optimal results do not depend on the block
-  bool doubled = rotate && pl.group != GAR_GROUP_XOR && P <= 1000 && pl.K > 1;
+  // Single-copy cyclic programs over 32 or more contributions run in 32-thread CTAs of at
+  // most 128 registers, with doubled pointer tables: a thread's P loads take long and
+  // vary, and a one-warp CTA frees its slot as soon as that warp is done instead of
+  // waiting for the slowest of eight.  GB300, against 256-thread CTAs: P = 127 x 8 MiB
+  // bf16 S = 14 0.351 -> 0.322 ms, P = 100 x 8 MiB bf16 0.270 -> 0.253, P = 40 x 12 MiB
+  // bf16 0.163 -> 0.151, P = 32 x 32 MiB bf16 0.334 -> 0.312, P = 127 x 8 MiB fp32
+  // 0.336 -> 0.327, P = 64 x 16 MiB fp32 0.324 -> 0.318, P = 64 x 16 MiB bf16 unchanged
+  // (0.314).  Without the doubled tables the 128-register cap spills (P = 127 bf16:
+  // 0.389 ms); fewer contributions gain nothing (P = 24 x 64 MiB fp32 0.467 ms either
+  // way) or lose (P = 8 x 256 MiB bf16 0.619 -> 0.627 ms).
+  const bool small_cta = pl.K == 1 && P >= 32 && P <= 1000 && rotate && pl.group != GAR_GROUP_XOR;
+  bool doubled = rotate && pl.group != GAR_GROUP_XOR && P <= 1000 && (pl.K > 1 || small_cta);
   if (const int d = tune_int("GAR_TUNE_DOUBLED", -1); d >= 0)
     doubled = d != 0 && rotate && pl.group != GAR_GROUP_XOR && P <= 1000;
   // bf16 programs with doubled pointer tables (below) run best with at most 8-byte
@@ -351,8 +362,8 @@ CodegenResult generate_fused_source(const gar_plan &pl, int threads_override, in
   while (W > 1 && pl.n / (uint64_t)W < 16384) W /= 2;
   if (int w = tune_int("GAR_TUNE_FUSED_W", 0))
     if (w > 0 && (w & (w - 1)) == 0 && w * elem_size(pl.dtype) <= 16) W = w;
-  const int minb = minb_override > 0 ? minb_override : tune_int("GAR_TUNE_FUSED_MINB", 0);
-  int nthr = threads_override > 0 ? threads_override : tune_int("GAR_TUNE_FUSED_THREADS", 256);
+  const int minb = minb_override > 0 ? minb_override : tune_int("GAR_TUNE_FUSED_MINB", small_cta ? 16 : 0);
+  int nthr = threads_override > 0 ? threads_override : tune_int("GAR_TUNE_FUSED_THREADS", small_cta ? 32 : 256);
   if (nthr < 32 || nthr > 1024 || nthr % 32 != 0) nthr = 256;
   const std::string bounds = minb > 0 ? fmt("__launch_bounds__(%d, %d)", nthr, minb)
                                       : fmt("__launch_bounds__(%d)", nthr);

@@ -302,8 +302,9 @@ def test_fused_program_size_limit():
 def test_fused_parameter_layout(P, n, S):
     """The generated kernel's gar_args must match the host packing in launch_fused_range:
     in[c P], out[c P], e_lo, e_hi, with c = 2 (tables stored twice) exactly for rotated
-    programs with several result copies (1 < K < P), else 1; kernels whose warps span
-    several blocks copy the tables to shared memory of the same size."""
+    programs with several result copies (1 < K < P) and for single-copy programs over 32
+    or more contributions (which also run in 32-thread CTAs), else 1; kernels whose warps
+    span several blocks copy the tables to shared memory of the same size."""
     plan = gar.gar_plan_create(P, n, "f32", "sum", S)
     src = gar.gar_plan_fused_source(plan)
     m = re.search(r"struct gar_args \{ const gar_io \*in\[(\d+)\]; gar_io \*out\[(\d+)\]; "
@@ -312,7 +313,9 @@ def test_fused_parameter_layout(P, n, S):
     c = int(m.group(1)) // P
     assert int(m.group(1)) == int(m.group(2)) == c * P and c in (1, 2)
     K = plan.info()["K"]
-    assert (c == 2) == (1 < K < P)
+    small_cta = K == 1 and 32 <= P <= 1000
+    assert (c == 2) == (1 < K < P or small_cta)
+    assert ("__launch_bounds__(32, 16)" in src) == small_cta
     if "__shared__" in src:
         assert K < P                          # only rotated programs are staged
         assert f"__shared__ const gar_io *s_in[{c * P}];" in src
