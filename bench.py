@@ -532,7 +532,7 @@ def measure_rows(gar, gar_inputs, stream, hbm_peak):
                "fused_combines_per_position": plan.info()["fused_combines"],
                "fused_width": plan.info()["fused_width"],
                "fused_regs": plan.info()["fused_regs"],
-               "fused_form": "breadth_first" if plan.info()["fused_form"] == 1 else "single"}
+               "fused_form": {0: "single", 1: "breadth_first", 2: "two_lane"}[plan.info()["fused_form"]]}
         if S in (7, 10, 14):
             gar.ensure_workspace(plan)
             ms_s = _time_loop(lambda: gar.gar_allreduce(plan, inp, "step", stream), 2, 1, stream)

@@ -129,7 +129,7 @@ typedef struct {
   int32_t fused_local_bytes; /* local (spill) bytes per thread of the loaded fused kernel */
   int32_t group;             /* GAR_GROUP_CYCLIC or GAR_GROUP_XOR */
   int32_t ring;              /* 1 for the Ring schedule (GAR_STEPS_RING) */
-  int32_t fused_form;        /* fused kernel the plan uses: GAR_FORM_SINGLE or GAR_FORM_BREADTH */
+  int32_t fused_form;        /* fused kernel the plan uses: GAR_FORM_SINGLE, _BREADTH or _SPLIT */
 } gar_plan_info;
 
 /* Values of gar_plan_info.fused_form.  GAR_FORM_SINGLE: each thread evaluates the whole
@@ -137,8 +137,13 @@ typedef struct {
  * evaluates it step by step for one element position, with paired fp32 adds; taken by
  * float sums with several result copies whose single-thread form would keep more than
  * 160 values alive per element position (large latency-optimal and near-latency-optimal
- * schedules, e.g. P = 127 at S = 7 and 8).  Both give the same bits. */
-enum { GAR_FORM_SINGLE = 0, GAR_FORM_BREADTH = 1 };
+ * schedules, e.g. P = 127 at S = 7 and 8).  GAR_FORM_SPLIT: two lanes of a warp share
+ * an element position, each evaluating the combines of half the placements and
+ * receiving the vectors a step moves across the halves by a warp shuffle; defined for
+ * latency-optimal cyclic schedules (every placement holds its own result copy) and
+ * taken only when forced (environment GAR_TUNE_FUSED_FORM=2): on GB300 it was slower
+ * than the breadth-first form.  All forms give the same bits. */
+enum { GAR_FORM_SINGLE = 0, GAR_FORM_BREADTH = 1, GAR_FORM_SPLIT = 2 };
 
 /* Creates a schedule for P virtual ranks of n elements each.
  * P: 1..GAR_MAX_P.  n: elements per rank (0 is allowed: every call is a no-op).

@@ -122,18 +122,28 @@ int check_fused_size(const gar_plan *pl) {
 // at S = 7 and 8: 254 and 192) are register-bound in that form and take the
 // breadth-first form (0.59 instead of 0.68 ms, and 0.47 instead of 0.56 ms, at P = 127 x
 // 8 MiB bf16 on GB300); every other plan takes the single-thread form.  GAR_TUNE_FUSED_FORM
-// (0 or 1) forces one form, for parity tests and launch-shape sweeps.
+// (0, 1 or 2) forces one form, for parity tests and launch-shape sweeps; the two-lane
+// form (2) exists for latency-optimal cyclic programs only and is never the default (P =
+// 127 x 8 MiB bf16 S = 7: 0.78 ms against 0.60 ms breadth-first; fp32: 0.416 against
+// 0.409 ms).
 int fused_form(const gar_plan &pl) {
   if (pl.K <= 1) return GAR_FORM_SINGLE;
   const char *ff = std::getenv("GAR_TUNE_FUSED_FORM");
-  if (ff && *ff) return std::atoi(ff) == 1 ? GAR_FORM_BREADTH : GAR_FORM_SINGLE;
+  if (ff && *ff) {
+    const int f = std::atoi(ff);
+    if (f == GAR_FORM_SPLIT) return split_form_applies(pl) ? GAR_FORM_SPLIT : GAR_FORM_BREADTH;
+    return f == GAR_FORM_BREADTH ? GAR_FORM_BREADTH : GAR_FORM_SINGLE;
+  }
   return (pl.op == GAR_SUM && pl.dtype != GAR_I32 && fused_peak_live(pl) > 160) ? GAR_FORM_BREADTH
                                                                                 : GAR_FORM_SINGLE;
 }
 
 CodegenResult fused_codegen(const gar_plan &pl) {
-  if (fused_form(pl) == GAR_FORM_BREADTH) return generate_fused_bf_source(pl);
-  return generate_fused_source(pl);
+  switch (fused_form(pl)) {
+    case GAR_FORM_BREADTH: return generate_fused_bf_source(pl);
+    case GAR_FORM_SPLIT: return generate_fused_split_source(pl);
+    default: return generate_fused_source(pl);
+  }
 }
 
 int compile_fused(gar_plan *pl) {
@@ -278,7 +288,10 @@ int launch_fused_range(gar_plan *pl, const void *const *in, void *const *out, ui
   std::memcpy(w, &e_lo, 8);
   std::memcpy(w + 8, &e_hi, 8);
   void *kargs[] = {args.data()};
-  const uint64_t items = (e_hi - e_lo) / pl->fused->width + 1;
+  // threads: one per vector of `width` positions, or two per position in groups of 16
+  // (two-lane form)
+  const uint64_t items = pl->fused->form == GAR_FORM_SPLIT ? (e_hi - e_lo + 15) / 16 * 32
+                                                           : (e_hi - e_lo) / pl->fused->width + 1;
   const int grid = grid_for(pl->fused, items);
   cudaError_t e = launch_generated(pl->fused, grid, kargs, stream);
   if (e != cudaSuccess) return cuda_fail(e, "fused kernel launch");

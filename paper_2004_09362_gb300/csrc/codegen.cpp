@@ -687,6 +687,248 @@ CodegenResult generate_fused_bf_source(const gar_plan &pl) {
 }
 
 
+// ---------------------------------------------------------------------------
+// Two-lane fused kernel for latency-optimal cyclic programs (K = P).
+//
+// The latency-optimal schedule keeps a q' and a q* vector at every placement (Sec.
+// "Latency-optimal version"): about 2P values per element position, which holds the
+// one-thread forms at 255 registers and spills.  Here two lanes of a warp share an
+// element position, lanes 0-15 and 16-31 of a warp serving the same 16 positions:
+//  * lane half A evaluates every combine at placements [0, m), m = ceil(P / 2), and
+//    half B the same code rotated by m placements, i.e. placements m .. m + m - 1 (mod
+//    P).  The program is invariant under rotation (copy s of the schedule is copy 0
+//    shifted by s), so one instruction stream serves both halves; for odd P the
+//    halves overlap in one placement, which B computes but does not store;
+//  * a step's shift by d moves some vectors across the halves' boundary.  Such an
+//    operand comes from the other half by one warp shuffle (xor 16): for the value A
+//    needs at placement g >= m, B holds it as its own value at g - m; B's counterpart
+//    is A's value at g - m + 1 (odd P) or g - m (even P).  Each half puts the value
+//    the other needs into the shuffle, so one shuffle serves both;
+//  * contributions and results go through pointer tables in shared memory indexed
+//    from each half's rank offset.
+// The combines and their operands are the schedule's, so the bits are too.
+// ---------------------------------------------------------------------------
+
+namespace {
+
+const char *kSplitHelpers = R"CUDA(
+static __device__ __forceinline__ gar_acc gar_xacc(gar_acc v) { return __shfl_xor_sync(0xffffffffu, v, 16); }
+static __device__ __forceinline__ gar_io gar_xio(gar_io v) {
+#if GAR_DTYPE == 1
+  return (gar_io)__shfl_xor_sync(0xffffffffu, (unsigned)v, 16);
+#else
+  return __shfl_xor_sync(0xffffffffu, v, 16);
+#endif
+}
+)CUDA";
+
+}  // namespace
+
+bool split_form_applies(const gar_plan &pl) {
+  const FusedProgram &fp = pl.prog;
+  const int P = pl.P;
+  if (pl.K != P || P < 4 || P > 1000 || pl.group == GAR_GROUP_XOR) return false;
+  const int nc = (int)fp.a.size();
+  if ((int)fp.place.size() != nc || (int)fp.star.size() != nc) return false;
+  // rotation by one placement maps the program onto itself
+  std::map<std::pair<int, int>, int> by_ops;
+  for (int k = 0; k < nc; ++k) by_ops[{fp.a[k], fp.b[k]}] = k;
+  std::vector<int> rot(P + nc, -1);
+  for (int j = 0; j < P; ++j) rot[j] = (j + 1) % P;
+  for (int k = 0; k < nc; ++k) {
+    const int ra = rot[fp.a[k]], rb = rot[fp.b[k]];
+    if (ra < 0 || rb < 0) return false;
+    auto it = by_ops.find({ra, rb});
+    if (it == by_ops.end() || fp.place[it->second] != (fp.place[k] + 1) % P ||
+        fp.star[it->second] != fp.star[k])
+      return false;
+    rot[P + k] = P + it->second;
+  }
+  for (int p = 0; p < P; ++p) {
+    const int v = fp.out[fp.origin[p]];
+    if (v < P || fp.place[v - P] != p) return false;
+  }
+  return true;
+}
+
+CodegenResult generate_fused_split_source(const gar_plan &pl) {
+  if (!split_form_applies(pl)) throw std::logic_error("program is not rotation invariant");
+  const FusedProgram &fp = pl.prog;
+  const int P = pl.P;
+  const int nc = (int)fp.a.size();
+  const int nv = P + nc;
+  const int m = (P + 1) / 2;
+  const bool odd = P % 2 == 1;
+  const bool sum_f = pl.op == GAR_SUM && pl.dtype != GAR_I32;
+  const bool bf16_sum = pl.op == GAR_SUM && pl.dtype == GAR_BF16;
+  auto plc = [&](int v) { return v < P ? v : (int)fp.place[v - P]; };
+
+  // rotations of every value by r placements, r = 1 .. P - 1 as needed
+  std::map<std::pair<int, int>, int> by_ops;
+  for (int k = 0; k < nc; ++k) by_ops[{fp.a[k], fp.b[k]}] = k;
+  auto rotation = [&](int r) {
+    std::vector<int> rt(nv);
+    for (int j = 0; j < P; ++j) rt[j] = (j + r) % P;
+    for (int k = 0; k < nc; ++k) rt[P + k] = P + by_ops.at({rt[fp.a[k]], rt[fp.b[k]]});
+    return rt;
+  };
+  const std::vector<int> rot_b = rotation(P - m);                 // what B sends: g - m
+  const std::vector<int> rot_a = rotation(odd ? P - m + 1 : P - m);  // what A sends
+
+  std::vector<int> level(nv, 0);
+  int maxlvl = 0;
+  for (int k = 0; k < nc; ++k) {
+    level[P + k] = 1 + std::max(level[fp.a[k]], level[fp.b[k]]);
+    maxlvl = std::max(maxlvl, level[P + k]);
+  }
+  // half A's combines, by level, in placement order (q* first at one placement)
+  std::vector<std::vector<int>> comb(maxlvl + 1);
+  for (int k = 0; k < nc; ++k)
+    if (fp.place[k] < m) comb[level[P + k]].push_back(k);
+  for (auto &cl : comb)
+    std::stable_sort(cl.begin(), cl.end(), [&](int x, int y) {
+      if (fp.place[x] != fp.place[y]) return fp.place[x] < fp.place[y];
+      return fp.star[x] > fp.star[y];
+    });
+
+  // Paired adds (float sums): two combines of a level at adjacent placements, same
+  // kind, whose operands are pairs in the same order, run as one __fadd2_rn.  Pairs:
+  // fp32 contributions 2k, 2k + 1; the results of a paired add; results at placements
+  // 2k, 2k + 1 of one kind; values received from the other half for such pairs.
+  const int pair_mode = tune_int("GAR_TUNE_SP_PAIR", 1);
+  std::vector<int> pair_hi(nv, -1), mate(nc, -1);
+  std::vector<char> is_hi(nc, 0);
+  if (sum_f && pair_mode > 0) {
+    if (pl.dtype == GAR_F32)
+      for (int j = 0; j + 1 < P; j += 2) pair_hi[j] = j + 1;
+    for (int L = 1; L <= maxlvl; ++L) {
+      const std::vector<int> &cl = comb[L];
+      std::map<std::pair<int, int>, int> at;  // (placement, star) -> combine
+      for (int c : cl) at[{fp.place[c], fp.star[c]}] = c;
+      for (int c1 : cl) {
+        if (mate[c1] >= 0 || is_hi[c1]) continue;
+        auto it = at.find({fp.place[c1] + 1, fp.star[c1]});
+        if (it == at.end()) continue;
+        const int c2 = it->second;
+        if (mate[c2] >= 0 || is_hi[c2] || fp.place[c2] >= m) continue;
+        const int a1 = fp.a[c1], b1 = fp.b[c1], a2 = fp.a[c2], b2 = fp.b[c2];
+        const bool leafbf = bf16_sum && (a1 < P || b1 < P || a2 < P || b2 < P);
+        if (leafbf) continue;
+        const bool ok = pair_mode == 2 || (pair_hi[a1] == a2 && pair_hi[b1] == b2);
+        if (!ok) continue;
+        mate[c1] = c2;
+        is_hi[c2] = 1;
+        pair_hi[P + c1] = P + c2;
+      }
+      for (int c : cl) {
+        const int v = P + c;
+        if (fp.place[c] % 2 != 0 || pair_hi[v] >= 0 || is_hi[c]) continue;
+        auto it = at.find({fp.place[c] + 1, fp.star[c]});
+        if (it == at.end() || is_hi[it->second] || pair_hi[P + it->second] >= 0) continue;
+        pair_hi[v] = P + it->second;
+      }
+    }
+  }
+
+  const int warps = std::max(1, std::min(16, tune_int("GAR_TUNE_SP_WARPS", 4)));
+  const int minb = std::max(1, tune_int("GAR_TUNE_SP_MINB", 3));
+  CodegenResult cg;
+  cg.width = 1;
+  cg.table_copies = 2;
+  cg.threads = 32 * warps;
+  cg.form = 2;
+  cg.kernel_name = fmt("gar_fusedsp_P%d_S%d_K%d_", P, pl.S, pl.K) + dtype_tag(pl.dtype) + "_" + op_tag(pl.op);
+
+  std::string s;
+  s += fmt("#define GAR_DTYPE %d\n#define GAR_OP %d\n", pl.dtype, pl.op);
+  s += "#define GAR_LDH \"" + tune_str("GAR_TUNE_LDH", ".cs") + "\"\n";
+  s += "#define GAR_STH \"" + tune_str("GAR_TUNE_STH", ".cs") + "\"\n";
+  s += kSkeleton;
+  s += kBFHelpers;
+  s += kSplitHelpers;
+  s += fmt("struct gar_args { const gar_io *in[%d]; gar_io *out[%d]; gar_u64 e_lo, e_hi; };\n", 2 * P, 2 * P);
+
+  std::string f = "static __device__ __forceinline__ void gar_eval_sp(const gar_io *const *tin, "
+                  "gar_io *const *tout, gar_u64 e, int hb, bool ok) {\n  (void)hb;\n";
+  std::vector<char> need_leaf(P, 0);
+  for (int L = 1; L <= maxlvl; ++L)
+    for (int k : comb[L])
+      for (int x : {fp.a[k], fp.b[k]})
+        if (x < P) need_leaf[x < m ? x : rot_a[x]] = need_leaf[x < m ? x : rot_b[x]] = 1;
+  for (int j = 0; j < m; ++j)
+    if (need_leaf[j]) f += fmt("  const gar_io l%d = gar_ldio(tin[%d] + e);\n", j, j);
+  // operand text; values at placements >= m arrive from the other half once
+  std::vector<char> got(nv, 0);
+  auto fetch = [&](int x) {
+    if (plc(x) < m || got[x]) return;
+    got[x] = 1;
+    const int vb = rot_b[x], va = rot_a[x];
+    if (x < P)
+      f += fmt("  const gar_io y%d = gar_xio(hb ? l%d : l%d);\n", x, vb, va);
+    else
+      f += fmt("  const gar_acc x%d = gar_xacc(hb ? v%d : v%d);\n", x, vb, va);
+  };
+  auto leaf = [&](int x) { return x < m ? fmt("l%d", x) : fmt("y%d", x); };
+  auto opnd = [&](int x) {
+    if (x < P) return "gar_wide(" + leaf(x) + ")";
+    return plc(x) < m ? fmt("v%d", x) : fmt("x%d", x);
+  };
+  for (int L = 1; L <= maxlvl; ++L) {
+    for (int k : comb[L]) {
+      if (is_hi[k]) continue;
+      const int v = P + k, a = fp.a[k], b = fp.b[k];
+      fetch(a);
+      fetch(b);
+      if (mate[k] >= 0) {
+        const int k2 = mate[k], v2 = P + k2;
+        fetch(fp.a[k2]);
+        fetch(fp.b[k2]);
+        f += fmt("  const float2 w%d = __fadd2_rn(make_float2(", v) + opnd(a) + ", " + opnd(fp.a[k2]) +
+             "), make_float2(" + opnd(b) + ", " + opnd(fp.b[k2]) + "));\n";
+        f += fmt("  const gar_acc v%d = w%d.x, v%d = w%d.y;\n", v, v, v2, v);
+      } else if (bf16_sum && (a < P || b < P)) {
+        const int lf = a < P ? a : b, other = a < P ? b : a;
+        f += fmt("  const gar_acc v%d = gar_addbf(", v) + leaf(lf) + ", " + opnd(other) + ");\n";
+      } else {
+        f += fmt("  const gar_acc v%d = gar_op(", v) + opnd(a) + ", " + opnd(b) + ");\n";
+      }
+    }
+  }
+  for (int p = 0; p < m; ++p) {
+    const int v = fp.out[fp.origin[p]];
+    const std::string st = fmt("gar_stio(tout[%d] + e, ", p) + opnd(v) + ");";
+    f += (odd && p == m - 1) ? "  if (ok && !hb) " + st + "\n" : "  if (ok) " + st + "\n";
+  }
+  f += "}\n";
+  s += f;
+
+  s += fmt("extern \"C\" __global__ void __launch_bounds__(%d, %d) ", cg.threads, minb) + cg.kernel_name +
+       "(const __grid_constant__ gar_args a) {\n";
+  s += fmt("  __shared__ const gar_io *s_in[%d];\n  __shared__ gar_io *s_out[%d];\n", 2 * P, 2 * P);
+  s += fmt("  for (int i = threadIdx.x; i < %d; i += blockDim.x) { s_in[i] = a.in[i]; s_out[i] = a.out[i]; }\n", 2 * P);
+  s += "  __syncthreads();\n";
+  // launched with programmatic stream serialisation: nothing is read before every
+  // earlier kernel on the stream has completed
+  s += "  asm volatile(\"griddepcontrol.wait;\" ::: \"memory\");\n";
+  s += "  const int lane = threadIdx.x & 31, hb = lane >> 4;\n";
+  s += fmt("  const gar_io *const *tin = s_in + (hb ? %d : 0);\n", m);
+  s += fmt("  gar_io *const *tout = s_out + (hb ? %d : 0);\n", m);
+  s += "  const gar_u64 npos = a.e_hi - a.e_lo;\n";
+  s += "  const gar_u64 gw = ((gar_u64)blockIdx.x * blockDim.x + threadIdx.x) >> 5;\n";
+  s += "  const gar_u64 nw = ((gar_u64)gridDim.x * blockDim.x) >> 5;\n";
+  // 16 element positions per warp; a ragged last group reads the last position again
+  // and stores nothing for the missing ones (every lane takes part in the shuffles)
+  s += "  for (gar_u64 base = gw * 16; base < npos; base += nw * 16) {\n";
+  s += "    const gar_u64 i = base + (gar_u64)(lane & 15);\n";
+  s += "    const bool ok = i < npos;\n";
+  s += "    gar_eval_sp(tin, tout, a.e_lo + (ok ? i : npos - 1), hb, ok);\n";
+  s += "  }\n";
+  s += "  asm volatile(\"griddepcontrol.launch_dependents;\" ::: \"memory\");\n}\n";
+  cg.source = s;
+  return cg;
+}
+
+
 CodegenResult generate_batched_source(const std::vector<const gar_plan *> &plans) {
   const gar_plan &p0 = *plans[0];
   int peak = 1;

@@ -142,6 +142,9 @@ CodegenResult generate_fused_source(const gar_plan &pl, int threads = 0, int min
 // The breadth-first form of the fused kernel (programs with many result copies), and
 // the peak number of live values of a plan's program in the single-thread form.
 CodegenResult generate_fused_bf_source(const gar_plan &pl);
+// two lanes per element position for rotation-invariant (latency-optimal cyclic) programs
+bool split_form_applies(const gar_plan &pl);
+CodegenResult generate_fused_split_source(const gar_plan &pl);
 int fused_peak_live(const gar_plan &pl);
 CodegenResult generate_batched_source(const std::vector<const gar_plan *> &plans);
 

@@ -21,7 +21,7 @@ GAR_SUM, GAR_MAX, GAR_MIN = 0, 1, 2
 GAR_STEP_FAITHFUL, GAR_FUSED, GAR_STEP_PERSISTENT = 0, 1, 2
 GAR_STEPS_BO, GAR_STEPS_LO, GAR_STEPS_RING = -1, -2, -3
 GAR_GROUP_CYCLIC, GAR_GROUP_XOR = 0, 1
-GAR_FORM_SINGLE, GAR_FORM_BREADTH = 0, 1
+GAR_FORM_SINGLE, GAR_FORM_BREADTH, GAR_FORM_SPLIT = 0, 1, 2
 GROUPS = {"cyclic": GAR_GROUP_CYCLIC, "xor": GAR_GROUP_XOR}
 GAR_MAX_P = 1024
 GAR_FUSED_MAX_OPS = 4096

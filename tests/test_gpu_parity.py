@@ -262,6 +262,22 @@ def test_breadth_first_form_every_step_count(P, n, dtype, op, monkeypatch):
         _assert_same(_run(plan, t, "fused"), G.allreduce(host, S, op, dtype), dtype, f"S={S}")
 
 
+@pytest.mark.parametrize("P,n", [(40, 40 * 97 + 13), (127, 127 * 40 + 19), (127, 3 * 127 + 5), (64, 64 * 33 + 1),
+                                 (5, 1000), (24, 24 * 16 + 15)])
+@pytest.mark.parametrize("dtype,op", [("f32", "sum"), ("bf16", "sum"), ("i32", "sum"), ("f32", "max"), ("bf16", "min")])
+def test_two_lane_form_latency_optimal(P, n, dtype, op, monkeypatch):
+    """The two-lane form forced on for the latency-optimal schedule, bit for bit against
+    the oracle; odd and even P, ragged n (the last warp's group of 16 positions is
+    partial)."""
+    monkeypatch.setenv("GAR_TUNE_FUSED_FORM", "2")
+    t = _np_inputs(P, n, dtype, seed=3 * P + n)
+    host = _to_host_list(t, dtype)
+    S = G.ceil_log2(P)
+    plan = gar.gar_plan_create(P, n, dtype, op, S)
+    assert gar.gar_plan_get_info(plan)["fused_form"] == gar.GAR_FORM_SPLIT
+    _assert_same(_run(plan, t, "fused"), G.allreduce(host, S, op, dtype), dtype, f"P={P} S={S}")
+
+
 def test_register_heavy_single_kernels_get_small_ctas():
     """Once prepared, a single-thread kernel of more than 128 registers runs in 64-thread
     CTAs capped at 168 registers; where that build spills more than 256 bytes per thread,
