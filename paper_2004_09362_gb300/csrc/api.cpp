@@ -187,10 +187,10 @@ int prepare_fused(gar_plan *pl) {
   const bool shape_forced = std::getenv("GAR_TUNE_FUSED_THREADS") || std::getenv("GAR_TUNE_FUSED_MINB");
   if (pl->fused->form != 0 || pl->fused->threads != 256 || shape_forced || pl->fused->regs <= 128)
     return GAR_OK;
-  auto build = [&](int threads, int minb, JitKernel **out) -> int {
+  auto build = [&](int threads, int minb, int fadd2, JitKernel **out) -> int {
     CodegenResult cg;
     try {
-      cg = generate_fused_source(*pl, threads, minb);
+      cg = generate_fused_source(*pl, threads, minb, fadd2);
     } catch (const std::exception &ex) {
       set_error(std::string("fused code generation: ") + ex.what());
       return GAR_EINVAL;
@@ -199,11 +199,22 @@ int prepare_fused(gar_plan *pl) {
     return jit_load(*out);
   };
   JitKernel *k = nullptr;
-  if ((rc = build(64, 5, &k))) return rc;
+  if ((rc = build(64, 5, -1, &k))) return rc;
   if (k->local_bytes > 256) {
     JitKernel *wide = nullptr;
-    if ((rc = build(32, 8, &wide))) return rc;
+    if ((rc = build(32, 8, -1, &wide))) return rc;
     if (wide->local_bytes < k->local_bytes) k = wide;
+  }
+  // bf16 kernels of 2-element vectors take paired fp32 adds only when the capped build is
+  // register-bound anyway (at the cap and spilling) and the paired build spills no more:
+  // then the pairs halve the adds at no cost in warps (P = 127 x 8 MiB S = 9: 0.405 ->
+  // 0.372 ms).  Elsewhere they cost registers: P = 100 S = 9 (128 -> 140 registers) 0.272
+  // -> 0.280 ms, P = 64 latency-optimal (39 -> 255) 0.339 -> 0.493 ms.
+  if (pl->dtype == GAR_BF16 && k->width == 2 && k->local_bytes > 0 && k->regs >= 168 &&
+      !std::getenv("GAR_TUNE_FADD2")) {
+    JitKernel *paired = nullptr;
+    if ((rc = build(k->threads, k->threads == 64 ? 5 : 8, 1, &paired))) return rc;
+    if (paired->local_bytes <= k->local_bytes) k = paired;
   }
   pl->fused = k;
   pl->fused_width = k->width;

@@ -334,7 +334,7 @@ std::string emit_block_of(const std::string &name, int P, uint64_t n) {
 
 }  // namespace
 
-CodegenResult generate_fused_source(const gar_plan &pl, int threads_override, int minb_override) {
+CodegenResult generate_fused_source(const gar_plan &pl, int threads_override, int minb_override, int fadd2_override) {
   const FusedProgram &fp = pl.prog;
   const int P = pl.P;
   Schedule sc = order_program(fp);
@@ -375,9 +375,11 @@ CodegenResult generate_fused_source(const gar_plan &pl, int threads_override, in
   std::string s;
   s += fmt("#define GAR_DTYPE %d\n#define GAR_OP %d\n", pl.dtype, pl.op);
   // paired fp32 adds over element positions for bf16 programs at W >= 4 (P = 127:
-  // S = 10 0.377 -> 0.360 ms, S = 11 0.354 -> 0.344 ms); fp32 programs and W = 2 were
-  // slower or spilled (P = 64 fp32, S = 8: 104 -> 255 registers)
-  s += fmt("#define GAR_FADD2 %d\n", tune_int("GAR_TUNE_FADD2", pl.dtype == GAR_BF16 && W >= 4) != 0 ? 1 : 0);
+  // S = 10 0.377 -> 0.360 ms, S = 11 0.354 -> 0.344 ms); fp32 programs were slower or
+  // spilled (P = 64 fp32, S = 8: 104 -> 255 registers); bf16 at W = 2 takes them only
+  // through fadd2_override, when the plan's prepared kernel is register-bound anyway
+  const int fadd2 = fadd2_override >= 0 ? fadd2_override : tune_int("GAR_TUNE_FADD2", pl.dtype == GAR_BF16 && W >= 4);
+  s += fmt("#define GAR_FADD2 %d\n", fadd2 != 0 ? 1 : 0);
   s += "#define GAR_LDH \"" + tune_str("GAR_TUNE_LDH", ".cs") + "\"\n";
   s += "#define GAR_STH \"" + tune_str("GAR_TUNE_STH", ".cs") + "\"\n";
   s += kSkeleton;

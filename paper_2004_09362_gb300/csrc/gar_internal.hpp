@@ -138,7 +138,7 @@ struct CodegenResult {
   int form = 0;          // fused kernels: 0 single-thread program, 1 breadth-first
 };
 // threads / minb > 0 override the CTA size and the minimum resident CTAs per SM
-CodegenResult generate_fused_source(const gar_plan &pl, int threads = 0, int minb = 0);
+CodegenResult generate_fused_source(const gar_plan &pl, int threads = 0, int minb = 0, int fadd2 = -1);
 // The breadth-first form of the fused kernel (programs with many result copies), and
 // the peak number of live values of a plan's program in the single-thread form.
 CodegenResult generate_fused_bf_source(const gar_plan &pl);
