@@ -170,7 +170,11 @@ template <> __device__ __forceinline__ void gar_store<4>(gar_io *p, const gar_ac
 // entry.  GAR_TUNE_FUSED_W: elements per thread-vector; GAR_TUNE_FUSED_MINB: minimum
 // resident CTAs per SM in __launch_bounds__; GAR_TUNE_LDH / GAR_TUNE_STH: cache-hint
 // suffix of the global loads / stores (default ".cs", streaming); GAR_TUNE_DOUBLED (0 or
-// 1): whether a rotated cyclic single-thread kernel stores its pointer tables twice.
+// 1): whether a rotated cyclic single-thread kernel stores its pointer tables twice;
+// GAR_TUNE_BF_ORDER / _BF_WARPS / _BF_MINB: combine order and CTA shape of the
+// breadth-first form; GAR_TUNE_SP_PAIR (0: no paired adds, 1: pairs of tracked operand
+// pairs, 2: any adjacent placements) / _SP_WARPS / _SP_MINB: the same for the two-lane
+// form.
 int tune_int(const char *name, int dflt) {
   const char *v = std::getenv(name);
   return (v && *v) ? std::atoi(v) : dflt;
