@@ -289,8 +289,8 @@ GAR_API int gar_allreduce_batched(gar_plan *const *plans, int nplans, const gar_
  * incomplete), or GAR_ECUDA.  GAR_OK if no persistent call ran. */
 GAR_API int gar_plan_status(gar_plan *plan);
 
-/* Barrier parameters of GAR_STEP_PERSISTENT (no counterpart in the paper).  spin_limit: polls (each an L2 round trip
- * plus a 64 ns sleep) a CTA makes at a grid barrier before it gives up (0 restores the
+/* Barrier parameters of GAR_STEP_PERSISTENT (no counterpart in the paper).  spin_limit: polls (each an L2 round trip,
+ * after the first 32 plus a 32 ns sleep) a CTA makes at a grid barrier before it gives up (0 restores the
  * default: 2^20 polls, roughly a second, or one poll per 256 bytes of memory traffic of
  * the plan's largest step if that is more -- a wait then outlasts that step many times
  * over).

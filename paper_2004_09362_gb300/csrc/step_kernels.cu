@@ -498,8 +498,8 @@ cudaError_t launch_pdl(void (*kernel)(Args), unsigned grid, gar_stream_t stream,
 // ---------------------------------------------------------------------------
 
 struct BarrierState {
-  unsigned int count;   // arrivals at the current barrier
-  unsigned int gen;     // barrier generation
+  unsigned int count;   // CTA arrivals since the launch began (zeroed before each launch)
+  unsigned int unused;
   int error;            // 1 once any CTA gave up waiting
   int error_launch;     // launch index after which the first timeout happened
 };
@@ -521,8 +521,10 @@ __device__ __forceinline__ unsigned ld_acquire_gpu(const unsigned *p) {
   asm volatile("ld.acquire.gpu.global.u32 %0, [%1];" : "=r"(v) : "l"(p) : "memory");
   return v;
 }
-__device__ __forceinline__ void st_release_gpu(unsigned *p, unsigned v) {
-  asm volatile("st.release.gpu.global.u32 [%0], %1;" ::"l"(p), "r"(v) : "memory");
+__device__ __forceinline__ unsigned atom_add_acq_rel_gpu(unsigned *p, unsigned v) {
+  unsigned old;
+  asm volatile("atom.add.acq_rel.gpu.global.u32 %0, [%1], %2;" : "=r"(old) : "l"(p), "r"(v) : "memory");
+  return old;
 }
 __device__ __forceinline__ int ld_relaxed_int(const int *p) {
   int v;
@@ -530,32 +532,32 @@ __device__ __forceinline__ int ld_relaxed_int(const int *p) {
   return v;
 }
 
-// Grid-wide barrier with a bounded wait.  Returns false (for the whole CTA) if this or
-// any other CTA timed out.
+// Grid-wide barrier number `launch` (0-based) with a bounded wait.  Every CTA adds one
+// to the arrival count with acquire-release semantics (release: the CTA's writes of the
+// step, ordered before it by __syncthreads, become visible with it; acquire: the CTA
+// that arrives last reads the others' writes, having seen all their arrivals in the add
+// itself) and polls the count with acquire loads until it reaches (launch + 1) *
+// expected, the arrivals of this and every earlier barrier of the launch.  The count
+// only grows within a launch, so no CTA resets it and the last arrival releases everyone
+// at once.  Returns false (for the whole CTA) if this or any other CTA timed out.
 __device__ bool grid_barrier(BarrierState *bar, unsigned expected, unsigned spin_limit, int launch) {
   __shared__ int s_ok;
-  __syncthreads();  // every thread's writes of this step precede thread 0's fence
+  __syncthreads();
   if (threadIdx.x == 0) {
     int ok = 1;
-    const unsigned g = ld_acquire_gpu(&bar->gen);
-    __threadfence();
-    const unsigned arrived = atomicAdd(&bar->count, 1u) + 1u;
-    if (arrived == expected) {
-      atomicExch(&bar->count, 0u);
-      __threadfence();
-      st_release_gpu(&bar->gen, g + 1u);
-    } else {
-      unsigned polls = 0;
-      while (ld_acquire_gpu(&bar->gen) == g) {
-        if (++polls >= spin_limit || ld_relaxed_int(&bar->error) != 0) {
-          ok = 0;
-          break;
-        }
-        __nanosleep(64);
+    const unsigned target = (unsigned)(launch + 1) * expected;
+    unsigned now = atom_add_acq_rel_gpu(&bar->count, 1u) + 1u;
+    unsigned polls = 0;
+    while (now < target) {
+      ++polls;
+      if (polls >= spin_limit || ((polls & 63u) == 0 && ld_relaxed_int(&bar->error) != 0)) {
+        ok = 0;
+        break;
       }
+      if (polls > 32) __nanosleep(32);
+      now = ld_acquire_gpu(&bar->count);
     }
     if (!ok && atomicCAS(&bar->error, 0, 1) == 0) bar->error_launch = launch;
-    __threadfence();
     s_ok = ok;
   }
   __syncthreads();
@@ -702,8 +704,14 @@ int launch_persistent_typed(const gar_plan &pl, void *const *rank, gar_stream_t 
   p.s.xor_group = pl.group == GAR_GROUP_XOR ? 1 : 0;
   const uint64_t maxblk = pl.q + (pl.rem ? 1 : 0);
   p.flat = maxblk < kFlatBelow ? 1 : 0;
+  // chunks as the per-step launches choose them for their largest step: small vectors
+  // drop to 8192 or 4096 elements so that the grid has work for every CTA it can hold
+  int max_ops = 1;
+  for (const Launch &ln : pl.launches) max_ops = std::max(max_ops, ln.nops);
   p.s.chunk = kChunk;
-  p.s.nchunks = (int)((maxblk + kChunk - 1) / kChunk);
+  const uint64_t min_items = 4 * (uint64_t)num_sms();
+  while (p.s.chunk > 4096 && ((maxblk + p.s.chunk - 1) / p.s.chunk) * pl.P * max_ops < min_items) p.s.chunk /= 2;
+  p.s.nchunks = (int)((maxblk + p.s.chunk - 1) / p.s.chunk);
   p.launches = static_cast<const LaunchDesc *>(pl.d_launches);
   p.step_bytes = pl.d_step_bytes;
   p.bar = static_cast<BarrierState *>(pl.d_barrier);
@@ -715,7 +723,16 @@ int launch_persistent_typed(const gar_plan &pl, void *const *rank, gar_stream_t 
   cudaError_t e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, fn, kThreads, 0);
   if (e != cudaSuccess || per_sm < 1) return cuda_fail(e == cudaSuccess ? cudaErrorInvalidConfiguration : e,
                                                        "persistent kernel occupancy");
-  const unsigned grid = (unsigned)(per_sm * num_sms());
+  // As many CTAs as the largest step has work items (one chunk of one block op, or 256
+  // element-major items), at most the co-resident maximum: a small Allreduce then waits
+  // at its barriers for a few CTAs instead of three per SM.
+  uint64_t need = 1;
+  for (const Launch &ln : pl.launches) {
+    const uint64_t items = p.flat ? ((uint64_t)ln.nops * pl.n + kThreads - 1) / kThreads
+                                  : (uint64_t)p.s.nchunks * (uint64_t)pl.P * (uint64_t)ln.nops;
+    need = std::max(need, items);
+  }
+  const unsigned grid = (unsigned)std::min<uint64_t>(need, (uint64_t)per_sm * (uint64_t)num_sms());
   void *args[] = {&p};
   e = cudaLaunchCooperativeKernel(fn, dim3(grid), dim3(kThreads), args, 0, (cudaStream_t)stream);
   if (e != cudaSuccess) return cuda_fail(e, "persistent kernel launch");
