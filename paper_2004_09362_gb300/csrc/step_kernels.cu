@@ -367,12 +367,24 @@ __device__ __forceinline__ void chunk_work(const StepArgs<MAXP> &a, const Launch
   }
   for (uint64_t e = vb + threadIdx.x; e < hi; e += blockDim.x) do1(e);
 
+  // The step's received bytes: summed over the warp, then over the CTA in shared memory,
+  // one atomic add per CTA into one of the step's 32 counter slots.  (Whether an op
+  // receives is the same for the whole CTA, so every thread takes this branch or none.)
   if (lv.bytes != nullptr && has_recv) {
+    __shared__ unsigned long long s_moved[kThreads / 32];
     unsigned long long m = moved;
 #pragma unroll
     for (int off = 16; off > 0; off >>= 1) m += __shfl_down_sync(0xffffffffu, m, off);
-    const unsigned long long esize = (op.recv_buf == BUF_RANK) ? sizeof(T) : sizeof(A);
-    if ((threadIdx.x & 31) == 0 && m) atomicAdd(lv.bytes + byte_slot(), m * esize);
+    if ((threadIdx.x & 31) == 0) s_moved[threadIdx.x >> 5] = m;
+    __syncthreads();
+    if (threadIdx.x == 0) {
+      unsigned long long t = 0;
+#pragma unroll
+      for (int w = 0; w < kThreads / 32; ++w) t += s_moved[w];
+      const unsigned long long esize = (op.recv_buf == BUF_RANK) ? sizeof(T) : sizeof(A);
+      if (t) atomicAdd(lv.bytes + blockIdx.x % STEP_BYTE_SLOTS, t * esize);
+    }
+    __syncthreads();  // s_moved is written again by the next work item of a persistent CTA
   }
 }
 
