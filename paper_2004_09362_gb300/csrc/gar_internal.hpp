@@ -108,7 +108,7 @@ struct gar_plan {
   // persistent step-faithful mode: launch table, barrier state, barrier parameters
   void *d_launches = nullptr;
   void *d_barrier = nullptr;
-  unsigned int barrier_spin_limit = 1u << 20;   // polls (each an L2 round trip + 64 ns); see default_spin_limit
+  unsigned int barrier_spin_limit = 1u << 20;   // polls (each an L2 round trip); see default_spin_limit
   unsigned int barrier_phantom = 0;
   bool ran_persistent = false;
   // pipelined host-buffer path: 3 streams (to device, kernel, to host) and events
