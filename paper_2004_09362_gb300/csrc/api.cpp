@@ -124,8 +124,8 @@ int check_fused_size(const gar_plan *pl) {
 // 8 MiB bf16 on GB300); every other plan takes the single-thread form.  GAR_TUNE_FUSED_FORM
 // (0, 1 or 2) forces one form, for parity tests and launch-shape sweeps; the two-lane
 // form (2) exists for latency-optimal cyclic programs only and is never the default (P =
-// 127 x 8 MiB bf16 S = 7: 0.78 ms against 0.60 ms breadth-first; fp32: 0.416 against
-// 0.409 ms).
+// 127 x 8 MiB bf16 S = 7: 0.78 ms against 0.60 ms breadth-first in one pass, 0.55 ms in
+// two; fp32: 0.416 against 0.409 ms in one pass).
 int fused_form(const gar_plan &pl) {
   if (pl.K <= 1) return GAR_FORM_SINGLE;
   const char *ff = std::getenv("GAR_TUNE_FUSED_FORM");

@@ -599,15 +599,25 @@ CodegenResult generate_fused_bf_source(const gar_plan &pl) {
     }
   }
 
-  // Launch shape, from P = 127 x 8 MiB bf16 on GB300: the widest programs (S = 7, 254
-  // live values) at 255 registers in 32-thread CTAs, 8 per SM (0.60 ms; 0.63 ms in
-  // 64-thread CTAs); the others at 168 registers (a third warp per sub-partition register
-  // file) in 128-thread CTAs, 3 per SM (S = 8, 192 live values: 0.464 ms; 0.473 ms in
-  // 64-thread CTAs, 0.48 ms in 32-thread ones, 0.56-0.60 ms at 255 or 128 registers).
+  // Launch shape, from P = 127 x 8 MiB bf16 on GB300: 168 registers (a third warp per
+  // sub-partition register file) in 128-thread CTAs, 3 per SM (S = 8, 192 live values:
+  // 0.464 ms; 0.473 ms in 64-thread CTAs, 0.48 ms in 32-thread ones, 0.56-0.60 ms at 255
+  // or 128 registers).  The widest programs (S = 7, 254 live values) evaluate their
+  // results in two passes (below), which brings them to 168 registers too: 0.552 ms,
+  // against 0.600 ms in one pass at 255 registers in 32-thread CTAs, 8 per SM.
   const int peak = order_program(fp).peak_live;
   const bool widest = peak >= 224;
-  const int warps = std::max(1, std::min(16, tune_int("GAR_TUNE_BF_WARPS", widest ? 1 : 4)));
-  const int minb = std::max(1, tune_int("GAR_TUNE_BF_MINB", widest ? 8 : 3));
+  const int warps = std::max(1, std::min(16, tune_int("GAR_TUNE_BF_WARPS", 4)));
+  const int minb = std::max(1, tune_int("GAR_TUNE_BF_MINB", 3));
+  // The results in G passes over contiguous placement groups, each pass evaluating only
+  // the values its group's results depend on: shared values are computed again in every
+  // pass that needs them, for fewer values alive at once.  The first pass copies the
+  // contributions to shared memory, where later passes read them (the first pass's
+  // results may already have overwritten them in place).  P = 127, S = 7: 1752
+  // combines in two passes instead of 1524, about 190 values alive instead of 286.
+  // S = 8 lost (0.466 -> 0.67-0.74 ms): its passes overlap more.  GAR_TUNE_BF_GROUPS
+  // overrides G.
+  const int groups = std::max(1, std::min(P, tune_int("GAR_TUNE_BF_GROUPS", widest ? 2 : 1)));
   // Pointer tables: the kernel parameters, indexed b + j (stored twice), while a warp's
   // 32 element positions share one block almost always (blocks of 32+ elements); with
   // shorter blocks the index differs across the lanes and the tables go to shared memory.
@@ -642,30 +652,77 @@ CodegenResult generate_fused_bf_source(const gar_plan &pl) {
   std::string f = "static __device__ __forceinline__ void gar_eval_bf(const gar_args &a, ";
   f += smem_tab ? "const gar_io *const *tin, gar_io *const *tout, " : "";
   f += "gar_u64 e, int b) {\n  (void)a; (void)b;\n";
-  for (int j = 0; j < P; ++j)
-    if (needs_leaf[j]) f += fmt("  const gar_io l%d = gar_ldio(", j) + tin + rank_of(j) + "] + e);\n";
-  auto opnd = [&](int x) { return x < P ? fmt("gar_wide(l%d)", x) : fmt("v%d", x); };
-  for (int L = 1; L <= maxlvl; ++L) {
-    for (int k : comb[L]) {
-      if (is_hi[k]) continue;
-      const int v = P + k, a = fp.a[k], b = fp.b[k];
-      if (mate[k] >= 0) {
-        const int k2 = mate[k], v2 = P + k2;
-        f += fmt("  const float2 w%d = __fadd2_rn(make_float2(", v) + opnd(a) + ", " + opnd(fp.a[k2]) +
-             "), make_float2(" + opnd(b) + ", " + opnd(fp.b[k2]) + "));\n";
-        f += fmt("  const gar_acc v%d = w%d.x, v%d = w%d.y;\n", v, v, v2, v);
-      } else if (bf16_sum && (a < P || b < P)) {
-        const int lf = a < P ? a : b, other = a < P ? b : a;
-        f += fmt("  const gar_acc v%d = gar_addbf(l%d, ", v, lf) + opnd(other) + ");\n";
-      } else {
-        f += fmt("  const gar_acc v%d = gar_op(", v) + opnd(a) + ", " + opnd(b) + ");\n";
+  if (groups > 1) {
+    s += fmt("#define GAR_BF_THREADS %d\n", cg.threads);
+    f += fmt("  __shared__ gar_io gar_sl_all[%d * GAR_BF_THREADS];\n", P);
+    f += "  gar_io *const gar_sl = gar_sl_all + threadIdx.x;\n";
+  }
+  std::vector<int> out_at(P);
+  {
+    std::vector<std::vector<int>> places_of(fp.K);
+    for (int p = 0; p < P; ++p) places_of[fp.origin[p]].push_back(p);
+    for (int sc = 0; sc < fp.K; ++sc)
+      for (int p : places_of[sc]) out_at[p] = fp.out[sc];
+  }
+  std::vector<int> lo_of(nc, -1);
+  for (int k = 0; k < nc; ++k)
+    if (mate[k] >= 0) lo_of[mate[k]] = k;
+  for (int g = 0; g < groups; ++g) {
+    const int p_lo = g * P / groups, p_hi = (g + 1) * P / groups;
+    std::vector<char> in_cone(nv, groups == 1 ? 1 : 0);
+    if (groups > 1) {
+      std::vector<int> st;
+      for (int p = p_lo; p < p_hi; ++p) st.push_back(out_at[p]);
+      while (!st.empty()) {
+        const int v = st.back();
+        st.pop_back();
+        if (in_cone[v]) continue;
+        in_cone[v] = 1;
+        if (v >= P) {
+          st.push_back(fp.a[v - P]);
+          st.push_back(fp.b[v - P]);
+        }
       }
     }
+    const std::string sfx = g == 0 ? "" : fmt("_%d", g);
+    for (int j = 0; j < P; ++j)
+      if (needs_leaf[j] && in_cone[j])
+        f += g == 0 ? fmt("  const gar_io l%d", j) + sfx + " = gar_ldio(" + tin + rank_of(j) + "] + e);\n"
+                    : fmt("  const gar_io l%d", j) + sfx + fmt(" = gar_sl[%d * GAR_BF_THREADS];\n", j);
+    if (g == 0 && groups > 1)
+      for (int j = 0; j < P; ++j)
+        if (needs_leaf[j]) f += fmt("  gar_sl[%d * GAR_BF_THREADS] = l%d;\n", j, j);
+    auto opnd = [&](int x) { return (x < P ? fmt("gar_wide(l%d", x) + sfx + ")" : fmt("v%d", x) + sfx); };
+    auto nm = [&](const char *f0, int v) { return fmt(f0, v) + sfx; };
+    for (int L = 1; L <= maxlvl; ++L) {
+      for (int k : comb[L]) {
+        const int v = P + k, a = fp.a[k], b = fp.b[k];
+        if (!in_cone[v]) continue;
+        if (is_hi[k] && in_cone[P + lo_of[k]]) continue;
+        if (mate[k] >= 0 && in_cone[P + mate[k]]) {
+          const int k2 = mate[k], v2 = P + k2;
+          f += "  const float2 " + nm("w%d", v) + " = __fadd2_rn(make_float2(" + opnd(a) + ", " + opnd(fp.a[k2]) +
+               "), make_float2(" + opnd(b) + ", " + opnd(fp.b[k2]) + "));\n";
+          f += "  const gar_acc " + nm("v%d", v) + " = " + nm("w%d", v) + ".x, " + nm("v%d", v2) + " = " +
+               nm("w%d", v) + ".y;\n";
+        } else if (bf16_sum && (a < P || b < P)) {
+          const int lf = a < P ? a : b, other = a < P ? b : a;
+          f += "  const gar_acc " + nm("v%d", v) + " = gar_addbf(" + nm("l%d", lf) + ", " + opnd(other) + ");\n";
+        } else {
+          f += "  const gar_acc " + nm("v%d", v) + " = gar_op(" + opnd(a) + ", " + opnd(b) + ");\n";
+        }
+      }
+    }
+    if (groups == 1) {
+      // result by result, each to every placement that holds it
+      std::vector<std::vector<int>> places_of(fp.K);
+      for (int p = 0; p < P; ++p) places_of[fp.origin[p]].push_back(p);
+      for (int sc = 0; sc < fp.K; ++sc)
+        for (int p : places_of[sc]) f += "  gar_stio(" + tout + rank_of(p) + "] + e, " + opnd(fp.out[sc]) + ");\n";
+    } else {
+      for (int p = p_lo; p < p_hi; ++p) f += "  gar_stio(" + tout + rank_of(p) + "] + e, " + opnd(out_at[p]) + ");\n";
+    }
   }
-  std::vector<std::vector<int>> places_of(fp.K);
-  for (int p = 0; p < P; ++p) places_of[fp.origin[p]].push_back(p);
-  for (int sc = 0; sc < fp.K; ++sc)
-    for (int p : places_of[sc]) f += "  gar_stio(" + tout + rank_of(p) + "] + e, " + opnd(fp.out[sc]) + ");\n";
   f += "}\n";
   s += f;
 

@@ -53,16 +53,21 @@ def test_selection():
         assert G.gar_plan_get_info(G.gar_plan_create(P, 4096, "f32", "sum", S))["fused_form"] == 0
 
 
-def test_every_combine_emitted_once():
-    """P = 127, S = 7: the 1524 combines are 2 x (paired adds) + single adds, and the
-    even-distance steps pair most of them."""
+def test_every_combine_emitted_once(monkeypatch):
+    """P = 127, S = 7 in one pass: the 1524 combines are 2 x (paired adds) + single adds,
+    and the even-distance steps pair most of them."""
+    monkeypatch.setenv("GAR_TUNE_BF_GROUPS", "1")
+    monkeypatch.setenv("GAR_TUNE_BF_WARPS", "1")
+    monkeypatch.setenv("GAR_TUNE_BF_MINB", "8")
     src, info = _bf_source(127, 4194304, "bf16", 7)
     body = re.search(r"void gar_eval_bf\(.*?\n\}\n", src, re.S).group(0)
     pairs = body.count("__fadd2_rn(make_float2(")
     singles = len(re.findall(r"const gar_acc v\d+ = gar_(?:addbf|op)\(", body))
     assert 2 * pairs + singles == info["fused_combines"] == 1524
     assert pairs >= 500
-    assert "__launch_bounds__(32, 8)" in src      # 254 live values: 255 registers
+    assert "__launch_bounds__(32, 8)" in src      # the shape forced above
+    monkeypatch.delenv("GAR_TUNE_BF_WARPS")
+    monkeypatch.delenv("GAR_TUNE_BF_MINB")
     src8, _ = _bf_source(127, 4194304, "bf16", 8)
     assert "__launch_bounds__(128, 3)" in src8    # 192 live values: 168 registers
 
@@ -75,7 +80,7 @@ def _bf16_round(x):
     return O.round_to_bf16(np.asarray(x, dtype=np.float32))
 
 
-def _run_generated(src, P, xs, dtype, op):
+def _run_generated(src, P, xs, dtype, op, in_place=False):
     """Evaluates gar_eval_bf for every element e of P rank vectors xs (numpy), returning
     the P output vectors.  The interpreter knows the few statement forms the generator
     emits; rank expressions are evaluated with the element's block b (mod P for the
@@ -106,36 +111,48 @@ def _run_generated(src, P, xs, dtype, op):
     if dtype == "i32":
         comb = {"sum": lambda a, c: np.int32((int(a) + int(c) + 2**31) % 2**32 - 2**31),
                 "max": lambda a, c: max(a, c), "min": lambda a, c: min(a, c)}[op]
-    out = [np.zeros_like(x) for x in xs]
+    out = xs if in_place else [np.zeros_like(x) for x in xs]
     lines = [ln.strip() for ln in body.split("\n") if ln.strip() and not ln.strip().startswith("(void)")]
+    N = r"(?:_\d+)?"   # pass suffix of the two-pass form
     for e in range(n):
         b = block_of(e)
         env = {}
+        shared = {}
 
         def val(tok):
             tok = tok.strip()
-            m = re.fullmatch(r"gar_wide\((l\d+)\)", tok)
+            m = re.fullmatch(r"gar_wide\((l\d+" + N + r")\)", tok)
             return env[m.group(1)] if m else env[tok]
 
         for ln in lines:
-            m = re.fullmatch(r"const gar_io (l\d+) = gar_ldio\((?:a\.in|tin)\[(.*)\] \+ e\);", ln)
+            if ln.startswith("__shared__ gar_io gar_sl_all[") or ln.startswith("gar_io *const gar_sl = "):
+                continue
+            m = re.fullmatch(r"gar_sl\[(\d+) \* GAR_BF_THREADS\] = (l\d+);", ln)
+            if m:
+                shared[int(m.group(1))] = env[m.group(2)]
+                continue
+            m = re.fullmatch(r"const gar_io (l\d+" + N + r") = gar_sl\[(\d+) \* GAR_BF_THREADS\];", ln)
+            if m:
+                env[m.group(1)] = shared[int(m.group(2))]
+                continue
+            m = re.fullmatch(r"const gar_io (l\d+" + N + r") = gar_ldio\((?:a\.in|tin)\[(.*)\] \+ e\);", ln)
             if m:
                 env[m.group(1)] = xs[rank(m.group(2), b)][e]
                 continue
-            m = re.fullmatch(r"const float2 (w\d+) = __fadd2_rn\(make_float2\((.*), (.*)\), make_float2\((.*), (.*)\)\);", ln)
+            m = re.fullmatch(r"const float2 (w\d+" + N + r") = __fadd2_rn\(make_float2\((.*), (.*)\), make_float2\((.*), (.*)\)\);", ln)
             if m:
                 env[m.group(1)] = (np.float32(val(m.group(2)) + val(m.group(4))),
                                    np.float32(val(m.group(3)) + val(m.group(5))))
                 continue
-            m = re.fullmatch(r"const gar_acc (v\d+) = (w\d+)\.x, (v\d+) = \2\.y;", ln)
+            m = re.fullmatch(r"const gar_acc (v\d+" + N + r") = (w\d+" + N + r")\.x, (v\d+" + N + r") = \2\.y;", ln)
             if m:
                 env[m.group(1)], env[m.group(3)] = env[m.group(2)]
                 continue
-            m = re.fullmatch(r"const gar_acc (v\d+) = gar_addbf\((l\d+), (.*)\);", ln)
+            m = re.fullmatch(r"const gar_acc (v\d+" + N + r") = gar_addbf\((l\d+" + N + r"), (.*)\);", ln)
             if m:
                 env[m.group(1)] = np.float32(env[m.group(2)] + val(m.group(3)))
                 continue
-            m = re.fullmatch(r"const gar_acc (v\d+) = gar_op\((.*), (.*)\);", ln)
+            m = re.fullmatch(r"const gar_acc (v\d+" + N + r") = gar_op\((.*), (.*)\);", ln)
             if m:
                 env[m.group(1)] = comb(val(m.group(2)), val(m.group(3)))
                 continue
@@ -177,6 +194,61 @@ def test_generated_code_reproduces_oracle(P, dtype, op, group):
             np.testing.assert_array_equal(np.asarray(got[x]).view(np.uint32 if dtype != "i32" else np.int32),
                                           np.asarray(want[x], dtype=got[x].dtype).view(np.uint32 if dtype != "i32" else np.int32),
                                           err_msg=f"P={P} S={S} rank {x}")
+
+
+@pytest.mark.parametrize("groups", [2, 3])
+@pytest.mark.parametrize("P,dtype,op,group", [(5, "f32", "sum", "cyclic"), (7, "bf16", "sum", "cyclic"),
+                                              (12, "f32", "sum", "cyclic"), (13, "bf16", "sum", "cyclic"),
+                                              (6, "f32", "max", "cyclic"), (8, "f32", "sum", "xor")])
+def test_generated_passes_reproduce_oracle(P, dtype, op, group, groups, monkeypatch):
+    """The form evaluated in several passes over placement groups (the default for the
+    widest programs, forced here on small ones): bit for bit against the oracle at every
+    step count with several result copies, ragged blocks.  The in-place Allreduce
+    overwrites contributions with results during the first pass, so later passes must
+    take the contributions from the shared-memory copy; the interpreter writes the
+    results into the same arrays it reads the contributions from, as the kernel does."""
+    monkeypatch.setenv("GAR_TUNE_BF_GROUPS", str(groups))
+    n = 3 * P + 2
+    xs = _inputs(P, n, dtype, seed=P * 7 + groups)
+    L = max(1, (P - 1).bit_length())
+    for S in range(L, 2 * L):
+        src, info = _bf_source(P, n, dtype, S, op, group)
+        assert "gar_sl[" in src
+        got = _run_generated(src, P, [x.copy() for x in xs], dtype, op, in_place=True)
+        want = O.allreduce(xs, S, op, dtype, group=group)
+        for x in range(P):
+            np.testing.assert_array_equal(np.asarray(got[x]).view(np.uint32 if dtype != "i32" else np.int32),
+                                          np.asarray(want[x], dtype=got[x].dtype).view(np.uint32 if dtype != "i32" else np.int32),
+                                          err_msg=f"P={P} S={S} groups={groups} rank {x}")
+
+
+def test_interpreter_catches_a_pass_reading_overwritten_contributions(monkeypatch):
+    """Planted mistake: later passes reading the contributions from global memory, where
+    the first pass has already stored results in place, break the comparison."""
+    monkeypatch.setenv("GAR_TUNE_BF_GROUPS", "2")
+    P, n, S = 7, 23, 3
+    xs = _inputs(P, n, "f32", 5)
+    src, _ = _bf_source(P, n, "f32", S)
+    bad = re.sub(r"const gar_io (l\d+_\d+) = gar_sl\[(\d+) \* GAR_BF_THREADS\];",
+                 lambda m: f"const gar_io {m.group(1)} = gar_ldio(a.in[{m.group(2)}] + e);", src)
+    assert bad != src
+    got = _run_generated(bad, P, [x.copy() for x in xs], "f32", "sum", in_place=True)
+    want = O.allreduce(xs, S, "sum", "f32")
+    assert any(not np.array_equal(got[x], want[x]) for x in range(P))
+
+
+def test_two_passes_for_the_widest_programs():
+    """P = 127, S = 7 evaluates its results in two passes (1752 combines: the shared
+    values are computed again) in 128-thread CTAs; S = 8 in one."""
+    src, info = _bf_source(127, 4194304, "bf16", 7)
+    body = re.search(r"void gar_eval_bf\(.*?\n\}\n", src, re.S).group(0)
+    pairs = body.count("__fadd2_rn(make_float2(")
+    singles = len(re.findall(r"const gar_acc v\d+(?:_\d+)? = gar_(?:addbf|op)\(", body))
+    assert 2 * pairs + singles == 1752
+    assert body.count("gar_ldio(") == 127 and body.count("gar_stio(") == 127
+    assert "__launch_bounds__(128, 3)" in src
+    src8, _ = _bf_source(127, 4194304, "bf16", 8)
+    assert "gar_sl[" not in src8
 
 
 def test_interpreter_catches_a_planted_mistake():
