@@ -609,15 +609,15 @@ CodegenResult generate_fused_bf_source(const gar_plan &pl) {
   const bool widest = peak >= 224;
   const int warps = std::max(1, std::min(16, tune_int("GAR_TUNE_BF_WARPS", 4)));
   const int minb = std::max(1, tune_int("GAR_TUNE_BF_MINB", 3));
-  // The results in G passes over contiguous placement groups, each pass evaluating only
-  // the values its group's results depend on: shared values are computed again in every
-  // pass that needs them, for fewer values alive at once.  The first pass copies the
+  // The results in G passes over contiguous groups of result copies, each pass evaluating
+  // only the values its group's results depend on: shared values are computed again in
+  // every pass that needs them, for fewer values alive at once.  The first pass copies the
   // contributions to shared memory, where later passes read them (the first pass's
   // results may already have overwritten them in place).  P = 127, S = 7: 1752
   // combines in two passes instead of 1524, about 190 values alive instead of 286.
   // S = 8 lost (0.466 -> 0.67-0.74 ms): its passes overlap more.  GAR_TUNE_BF_GROUPS
   // overrides G.
-  const int groups = std::max(1, std::min(P, tune_int("GAR_TUNE_BF_GROUPS", widest ? 2 : 1)));
+  const int groups = std::max(1, std::min(fp.K, tune_int("GAR_TUNE_BF_GROUPS", widest ? 2 : 1)));
   // Pointer tables: the kernel parameters, indexed b + j (stored twice), while a warp's
   // 32 element positions share one block almost always (blocks of 32+ elements); with
   // shorter blocks the index differs across the lanes and the tables go to shared memory.
@@ -657,22 +657,18 @@ CodegenResult generate_fused_bf_source(const gar_plan &pl) {
     f += fmt("  __shared__ gar_io gar_sl_all[%d * GAR_BF_THREADS];\n", P);
     f += "  gar_io *const gar_sl = gar_sl_all + threadIdx.x;\n";
   }
-  std::vector<int> out_at(P);
-  {
-    std::vector<std::vector<int>> places_of(fp.K);
-    for (int p = 0; p < P; ++p) places_of[fp.origin[p]].push_back(p);
-    for (int sc = 0; sc < fp.K; ++sc)
-      for (int p : places_of[sc]) out_at[p] = fp.out[sc];
-  }
   std::vector<int> lo_of(nc, -1);
   for (int k = 0; k < nc; ++k)
     if (mate[k] >= 0) lo_of[mate[k]] = k;
+  std::vector<std::vector<int>> places_of(fp.K);
+  for (int p = 0; p < P; ++p) places_of[fp.origin[p]].push_back(p);
   for (int g = 0; g < groups; ++g) {
-    const int p_lo = g * P / groups, p_hi = (g + 1) * P / groups;
+    // group g: result copies [c_lo, c_hi), each stored to every placement that holds it
+    const int c_lo = g * fp.K / groups, c_hi = (g + 1) * fp.K / groups;
     std::vector<char> in_cone(nv, groups == 1 ? 1 : 0);
     if (groups > 1) {
       std::vector<int> st;
-      for (int p = p_lo; p < p_hi; ++p) st.push_back(out_at[p]);
+      for (int sc = c_lo; sc < c_hi; ++sc) st.push_back(fp.out[sc]);
       while (!st.empty()) {
         const int v = st.back();
         st.pop_back();
@@ -685,8 +681,9 @@ CodegenResult generate_fused_bf_source(const gar_plan &pl) {
       }
     }
     const std::string sfx = g == 0 ? "" : fmt("_%d", g);
+    // the first pass loads every contribution (later passes read its shared-memory copy)
     for (int j = 0; j < P; ++j)
-      if (needs_leaf[j] && in_cone[j])
+      if (needs_leaf[j] && (in_cone[j] || g == 0))
         f += g == 0 ? fmt("  const gar_io l%d", j) + sfx + " = gar_ldio(" + tin + rank_of(j) + "] + e);\n"
                     : fmt("  const gar_io l%d", j) + sfx + fmt(" = gar_sl[%d * GAR_BF_THREADS];\n", j);
     if (g == 0 && groups > 1)
@@ -713,15 +710,8 @@ CodegenResult generate_fused_bf_source(const gar_plan &pl) {
         }
       }
     }
-    if (groups == 1) {
-      // result by result, each to every placement that holds it
-      std::vector<std::vector<int>> places_of(fp.K);
-      for (int p = 0; p < P; ++p) places_of[fp.origin[p]].push_back(p);
-      for (int sc = 0; sc < fp.K; ++sc)
-        for (int p : places_of[sc]) f += "  gar_stio(" + tout + rank_of(p) + "] + e, " + opnd(fp.out[sc]) + ");\n";
-    } else {
-      for (int p = p_lo; p < p_hi; ++p) f += "  gar_stio(" + tout + rank_of(p) + "] + e, " + opnd(out_at[p]) + ");\n";
-    }
+    for (int sc = c_lo; sc < c_hi; ++sc)
+      for (int p : places_of[sc]) f += "  gar_stio(" + tout + rank_of(p) + "] + e, " + opnd(fp.out[sc]) + ");\n";
   }
   f += "}\n";
   s += f;
