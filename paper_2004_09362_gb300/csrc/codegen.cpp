@@ -615,8 +615,8 @@ CodegenResult generate_fused_bf_source(const gar_plan &pl) {
   // contributions to shared memory, where later passes read them (the first pass's
   // results may already have overwritten them in place).  P = 127, S = 7: 1752
   // combines in two passes instead of 1524, about 190 values alive instead of 286.
-  // S = 8 lost (0.466 -> 0.67-0.74 ms): its passes overlap more.  GAR_TUNE_BF_GROUPS
-  // overrides G.
+  // S = 8 (64 copies) lost: 996 combines in two passes, 158 values alive instead of 190,
+  // 0.477-0.516 ms against 0.464 in one.  GAR_TUNE_BF_GROUPS overrides G.
   const int groups = std::max(1, std::min(fp.K, tune_int("GAR_TUNE_BF_GROUPS", widest ? 2 : 1)));
   // Pointer tables: the kernel parameters, indexed b + j (stored twice), while a warp's
   // 32 element positions share one block almost always (blocks of 32+ elements); with
