@@ -222,6 +222,23 @@ def test_generated_passes_reproduce_oracle(P, dtype, op, group, groups, monkeypa
                                           err_msg=f"P={P} S={S} groups={groups} rank {x}")
 
 
+@pytest.mark.parametrize("dtype", ["bf16", "f32"])
+def test_p127_latency_optimal_kernel_reproduces_oracle(dtype):
+    """The kernel text the P = 127 latency-optimal plan runs by default (breadth-first,
+    two passes; it does not depend on n for an unrotated program, so a 6-element plan
+    has the same text as the 8 MiB one), interpreted in place against the oracle."""
+    P, n, S = 127, 6, 7
+    xs = _inputs(P, n, dtype, seed=11)
+    src = G.gar_plan_fused_source(G.gar_plan_create(P, n, dtype, "sum", S))
+    assert src == G.gar_plan_fused_source(G.gar_plan_create(P, 4194304, dtype, "sum", S))
+    assert "gar_sl[" in src
+    got = _run_generated(src, P, [x.copy() for x in xs], dtype, "sum", in_place=True)
+    want = O.allreduce(xs, S, "sum", dtype)
+    for x in range(P):
+        np.testing.assert_array_equal(np.asarray(got[x]).view(np.uint32),
+                                      np.asarray(want[x], dtype=np.float32).view(np.uint32), err_msg=f"rank {x}")
+
+
 def test_interpreter_catches_a_pass_reading_overwritten_contributions(monkeypatch):
     """Planted mistake: later passes reading the contributions from global memory, where
     the first pass has already stored results in place, break the comparison."""
