@@ -168,6 +168,20 @@ def test_p127_exchange_count():
     assert body.count("gar_ldio(tin[") == 64 and body.count("gar_stio(tout[") == 64
 
 
+def test_p127_kernel_reproduces_oracle():
+    """The P = 127 latency-optimal two-lane kernel (the shape the GPU sweeps ran),
+    interpreted for both halves against the oracle."""
+    P, n, S = 127, 6, 7
+    xs = _inputs(P, n, "bf16", seed=5)
+    src, info = _split_source(P, n, "bf16", S)
+    assert info["fused_form"] == G.GAR_FORM_SPLIT
+    got = _run_split(src, P, xs, "bf16", "sum")
+    want = O.allreduce(xs, S, "sum", "bf16")
+    for x in range(P):
+        np.testing.assert_array_equal(_bits(got[x], "bf16"), _bits(np.asarray(want[x], dtype=np.float32), "bf16"),
+                                      err_msg=f"rank {x}")
+
+
 def test_interpreter_catches_a_planted_mistake():
     """Swapping the two sources of one exchange breaks the comparison."""
     P, n, S = 7, 17, 3
