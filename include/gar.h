@@ -134,10 +134,11 @@ typedef struct {
 
 /* Values of gar_plan_info.fused_form.  GAR_FORM_SINGLE: each thread evaluates the whole
  * program result by result for 1..8 element positions.  GAR_FORM_BREADTH: each thread
- * evaluates it step by step for one element position, with paired fp32 adds; taken by
- * float sums with several result copies whose single-thread form would keep more than
- * 160 values alive per element position (large latency-optimal and near-latency-optimal
- * schedules, e.g. P = 127 at S = 7 and 8).  GAR_FORM_SPLIT: two lanes of a warp share
+ * evaluates it step by step for one element position, with paired fp32 adds (the widest
+ * programs in two passes over halves of the result copies, recomputing the values both
+ * halves need); taken by float sums with several result copies whose single-thread form
+ * would keep more than 160 values alive per element position (large latency-optimal and
+ * near-latency-optimal schedules, e.g. P = 127 at S = 7 and 8).  GAR_FORM_SPLIT: two lanes of a warp share
  * an element position, each evaluating the combines of half the placements and
  * receiving the vectors a step moves across the halves by a warp shuffle; defined for
  * latency-optimal cyclic schedules (every placement holds its own result copy) and
