@@ -300,3 +300,34 @@ def test_breadth_first_kernels_compile(P):
             G.gar_plan_compile(G.gar_plan_create_group(P, 1000, "f32", "sum", L, "xor"), "fused")
     _with_form(1, go)
 
+
+
+@pytest.mark.parametrize("groups", [2, 3])
+def test_pass_kernels_compile(groups, monkeypatch):
+    """NVRTC compiles the several-pass form (shared-memory copy of the contributions,
+    suffixed values) for rotated and unrotated programs, sums and max."""
+    monkeypatch.setenv("GAR_TUNE_FUSED_FORM", "1")
+    monkeypatch.setenv("GAR_TUNE_BF_GROUPS", str(groups))
+    for P in (5, 12, 33):
+        L = max(1, (P - 1).bit_length())
+        for dtype in ("f32", "bf16"):
+            for op in ("sum", "max"):
+                for S in (L, L + 1):
+                    G.gar_plan_compile(G.gar_plan_create(P, 4 * P + 3, dtype, op, S), "fused")
+
+
+def test_default_p127_latency_optimal_kernel_compiles():
+    """The P = 127 latency-optimal default (two passes) compiles for sm_103a."""
+    G.gar_plan_compile(G.gar_plan_create(127, 4096, "bf16", "sum", 7), "fused")
+
+
+def test_fused_form_matches_generated_kernel():
+    """gar_plan_info.fused_form names the kernel the plan's source defines."""
+    for P in (5, 24, 64, 127):
+        L = max(1, (P - 1).bit_length())
+        for S in range(L, 2 * L + 1):
+            pl = G.gar_plan_create(P, 4096, "bf16", "sum", S)
+            form = G.gar_plan_get_info(pl)["fused_form"]
+            src = G.gar_plan_fused_source(pl)
+            assert ("gar_fusedbf_" in src) == (form == G.GAR_FORM_BREADTH), (P, S)
+            assert ("gar_fused_P" in src) == (form == G.GAR_FORM_SINGLE), (P, S)
